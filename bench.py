@@ -1,0 +1,443 @@
+#!/usr/bin/env python3
+"""Sparse-FFN decode benchmark (PrunePath hot path on GB300).
+
+Workload (default): the Llama-2-7B-shaped SwiGLU FFN, bf16, d=4096,
+d_ff=11008, E=172 experts of 64 neurons, 32 stacked layers, batch-1 decode,
+p = 0.7.  One step = one token through all 32 layers: for each layer one
+``pp_layer`` call (router GEMV, softmax, sort, cumulative-mass cut, sparse
+SwiGLU FFN over the selected experts).  Synthetic weights/inputs (seeded
+torch CUDA generator, recipe in paper_2605_28283_gb300/workloads.py); each
+layer cycles through a pool of pre-drawn token vectors so the expert choice
+changes every step.  The 32 launches of a step are one CUDA graph; L2 is
+flushed (256 MiB write) between steps, outside the timed events.
+
+Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle
+instead (the reference arm of this build: a plain fp64 implementation).
+"""
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "sparse-FFN decode tokens/s; HBM GB/s on touched expert bytes vs peak"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama2_7b_decode")
+    ap.add_argument("--p", type=float, default=0.7)
+    ap.add_argument("--batch", type=int, default=1)
+    ap.add_argument("--pool", type=int, default=16, help="distinct token vectors per layer")
+    ap.add_argument("--sweep", default="0.3,0.5,0.7,0.9,1.0", help="p values for the sweep ('' = none)")
+    ap.add_argument("--sweep-steps", type=int, default=400)
+    ap.add_argument("--no-flush", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--seed", type=int, default=0)
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            pk = json.load(f)
+        return float(pk["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+# --------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "50"], stdout=self.out,
+                stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.out.close()
+        rows = []
+        for line in open(self.path):
+            parts = [s.strip() for s in line.split(",")]
+            if len(parts) != 7:
+                continue
+            try:
+                rows.append((float(parts[0]), float(parts[1]), parts[3:]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i, v in enumerate(r) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# -------------------------------------------------------------- workload
+def make_layers(w, args, device):
+    import torch
+    from paper_2605_28283_gb300 import workloads as wl
+    layers = []
+    for l in range(w.n_layers):
+        t = wl.device_layer(w, args.batch, args.seed, l, device, n_token_sets=args.pool)
+        t["y"] = torch.empty((args.batch, w.d_model), dtype=t["x"].dtype, device=device)
+        layers.append(t)
+    return layers
+
+
+def capture_graphs(pp, desc, layers, p, B, pool, ws, stream):
+    import torch
+    graphs = []
+    with torch.cuda.stream(stream):
+        for i in range(pool):  # warm the launch path once per pool entry outside capture
+            for L in layers:
+                pp.pp_layer(desc, L["x"][i], B, L["Wr"], L["Wg"], L["Wu"], L["Wd"], p, None, L["y"], ws,
+                            stream=stream)
+        stream.synchronize()
+        for i in range(pool):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for L in layers:
+                    pp.pp_layer(desc, L["x"][i], B, L["Wr"], L["Wg"], L["Wu"], L["Wd"], p, None, L["y"],
+                                ws, stream=stream)
+            graphs.append(g)
+    return graphs
+
+
+def time_graphs(graphs, steps, warmup, flush_buf, stream):
+    """Per-step CUDA-event timing on `stream`; L2 flushed between steps."""
+    import torch
+    with torch.cuda.stream(stream):
+        for i in range(warmup):
+            graphs[i % len(graphs)].replay()
+        stream.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(steps)]
+        for i in range(steps):
+            if flush_buf is not None:
+                flush_buf.add_(1)
+            ev[i][0].record(stream)
+            graphs[i % len(graphs)].replay()
+            ev[i][1].record(stream)
+        stream.synchronize()
+    return [a.elapsed_time(b) for a, b in ev]  # ms
+
+
+def selection_stats(pp, desc, layers, w, p, B, pool, ws):
+    """k per (pool entry, layer, token) via pp_route on the same inputs."""
+    import torch
+    ks = torch.empty((pool, len(layers), B), dtype=torch.int64)
+    union = torch.empty((pool, len(layers)), dtype=torch.int64)
+    sel = pp.Selection.empty(B, w.n_experts, "cuda", with_logits=False)
+    for i in range(pool):
+        for l, L in enumerate(layers):
+            pp.pp_route(desc, L["x"][i], B, L["Wr"], p, sel, ws)
+            c = sel.counts.cpu()
+            ks[i, l] = c.long()
+            ids = sel.ids.cpu()
+            u = set()
+            for t in range(B):
+                u.update(ids[t, :int(c[t])].tolist())
+            union[i, l] = len(u)
+    return ks, union
+
+
+def layer_bytes(w, B, n_union):
+    """Algorithmic HBM bytes of one pp_layer launch: W_r, the union of the
+    selected expert blocks (gate+up rows and down column block), x and y."""
+    esz = 2 if w.dtype == "bf16" else 4
+    mats = 3 if w.gated else 2
+    router = w.n_experts * w.d_model * esz
+    expert = mats * 64 * w.d_model * esz
+    act = 2 * B * w.d_model * esz
+    return router + n_union * expert + act, n_union * expert
+
+
+def kernel_traffic(workload, p):
+    """DRAM bytes per launch of the layer kernel from a committed ncu summary,
+    valid only while the kernel sources are unchanged."""
+    path = os.path.join(ROOT, "profiles", "decode_layer_traffic.json")
+    try:
+        rec = json.load(open(path))
+    except Exception:
+        return None
+    if rec.get("sources_sha") != sources_sha():
+        return None
+    ent = rec.get("entries", {}).get("%s@%g" % (workload, p))
+    return None if ent is None else ent.get("dram_bytes_per_launch")
+
+
+def sources_sha():
+    h = hashlib.sha256()
+    d = os.path.join(ROOT, "paper_2605_28283_gb300", "csrc")
+    for n in sorted(os.listdir(d)):
+        with open(os.path.join(d, n), "rb") as f:
+            h.update(n.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+# ------------------------------------------------------------ CPU oracle
+def run_oracle_sample(w, seconds, seed, host_layers=None, p=0.7, B=1):
+    """Times the oracle (as it stands) on a bounded sample of the workload:
+    whole-layer calls (logits, selection, sparse FFN) for B tokens, over a
+    few layers, repeated until `seconds` of CPU work; scaled to tokens/s of
+    the full L-layer model."""
+    import numpy as np
+    import oracle
+    from paper_2605_28283_gb300 import workloads as wl
+    oracle.load()
+    n_layers = 2 if host_layers is None else len(host_layers)
+    if host_layers is None:
+        host_layers = [wl.host_layer(w, B, seed=seed, layer=l) for l in range(n_layers)]
+    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    calls = 0
+    t0 = time.perf_counter()
+    while True:
+        for L in host_layers:
+            oracle.layer(L.x, L.Wr, L.Wg, L.Wu, L.Wd, float(np.float32(p)), w.act, "sigmoid")
+            calls += 1
+        el = time.perf_counter() - t0
+        if el >= seconds:
+            break
+    per_layer = el / calls
+    tok_s = B / (per_layer * w.n_layers)
+    return {"value": tok_s, "unit": "tokens/s", "cores": min(threads, B) if B > 0 else 1, "kind": "oracle",
+            "sample": "%d calls of one layer x %d token(s) over %d distinct layers (%.1f s CPU); "
+                      "scaled to %d layers" % (calls, B, n_layers, el, w.n_layers)}
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    from paper_2605_28283_gb300 import workloads as wl
+    w = wl.WORKLOADS[args.workload]
+    if rank != 0:
+        return
+    # Each step is one bounded sample (a single layer call), scaled to the
+    # full model; the whole run stays within a few minutes.
+    import numpy as np
+    import oracle
+    oracle.load()
+    L = wl.host_layer(w, args.batch, seed=args.seed, layer=0)
+    p = float(np.float32(args.p))
+    for _ in range(max(1, min(args.warmup, 3))):
+        oracle.layer(L.x, L.Wr, L.Wg, L.Wu, L.Wd, p, w.act, "sigmoid")
+    steps = max(1, min(args.steps, 200))
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        oracle.layer(L.x, L.Wr, L.Wg, L.Wu, L.Wd, p, w.act, "sigmoid")
+    el = time.perf_counter() - t0
+    per_step_model = el / steps * w.n_layers
+    value = args.batch / per_step_model
+    cores = 1
+    out = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus, "steps": steps,
+           "warmup": args.warmup, "ms_per_step": per_step_model * 1e3, "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "impl": "reference",
+           "config": {"workload": w.name, "d_model": w.d_model, "d_ff": w.d_ff, "n_experts": w.n_experts,
+                      "layers": w.n_layers, "batch": args.batch, "p": args.p},
+           "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                            "sample": "%d single-layer calls (layer 0) x %d token(s), scaled to %d layers"
+                                      % (steps, args.batch, w.n_layers)},
+           "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out))
+
+
+# ------------------------------------------------------------------ main
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    import numpy as np
+    import torch
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    device = torch.device("cuda", torch.cuda.current_device())
+    from paper_2605_28283_gb300 import binding as pp
+    from paper_2605_28283_gb300 import workloads as wl
+    pp.load()
+    w = wl.WORKLOADS[args.workload]
+    B = args.batch
+    desc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act)
+    stream = torch.cuda.Stream()
+    ws = pp.alloc_workspace(desc, B)
+    layers = make_layers(w, args, device)
+    flush = None if args.no_flush else torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=device)
+    torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+
+    def max_over_ranks(v):
+        if world == 1:
+            return v
+        t = torch.tensor([v], dtype=torch.float64, device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        return float(t.item())
+
+    # ---- headline: p = args.p
+    pf = float(np.float32(args.p))
+    graphs = capture_graphs(pp, desc, layers, pf, B, args.pool, ws, stream)
+    sampler = ClockSampler(local)
+    barrier()
+    sampler.start()
+    times = time_graphs(graphs, args.steps, args.warmup, flush, stream)
+    barrier()
+    clocks = sampler.stop()
+    total_ms = max_over_ranks(sum(times))
+    status = pp.pp_get_device_status(ws)
+    if status != pp.PP_OK:
+        raise SystemExit("device status: %s" % pp.status_name(status))
+    ms_per_step = total_ms / args.steps
+    value = world * B * args.steps / (total_ms / 1e3)
+
+    # bytes per step from the actual selections of the pool entries
+    ks, union = selection_stats(pp, desc, layers, w, pf, B, args.pool, ws)
+    step_ids = np.arange(args.steps) % args.pool
+    tot_b, exp_b = 0.0, 0.0
+    for i in range(args.pool):
+        n_i = int((step_ids == i).sum())
+        for l in range(w.n_layers):
+            a, e = layer_bytes(w, B, int(union[i, l]))
+            tot_b += n_i * a
+            exp_b += n_i * e
+    seconds = sum(times) / 1e3
+    launches = args.steps * w.n_layers
+    per_launch_ms = sum(times) / launches   # step time / L: includes the in-graph launch gaps
+    bytes_per_launch = tot_b / launches
+    peak, peak_kind = load_peaks()
+    achieved = bytes_per_launch / (per_launch_ms / 1e3) / 1e9
+    expert_gbs = exp_b / seconds / 1e9
+    k_mean = float(ks.float().mean())
+    s_ffn = 1.0 - k_mean / w.n_experts
+
+    # ---- p sweep (same kernels), speedup vs dense p >= 1
+    sweep = {}
+    if args.sweep:
+        for ps in [float(v) for v in args.sweep.split(",") if v]:
+            psf = float(np.float32(ps))
+            gs = capture_graphs(pp, desc, layers, psf, B, args.pool, ws, stream)
+            tm = time_graphs(gs, args.sweep_steps, 5, flush, stream)
+            kk, un = selection_stats(pp, desc, layers, w, psf, B, args.pool, ws)
+            sid = np.arange(args.sweep_steps) % args.pool
+            eb = sum(int((sid == i).sum()) * layer_bytes(w, B, int(un[i, l]))[1]
+                     for i in range(args.pool) for l in range(w.n_layers))
+            tb = sum(int((sid == i).sum()) * layer_bytes(w, B, int(un[i, l]))[0]
+                     for i in range(args.pool) for l in range(w.n_layers))
+            sec = sum(tm) / 1e3
+            sweep["%g" % ps] = {"tokens_per_s": B * args.sweep_steps / sec, "ms_per_step": sum(tm) / args.sweep_steps,
+                                "k_mean": float(kk.float().mean()), "s_ffn": 1 - float(kk.float().mean()) / w.n_experts,
+                                "expert_gbs": eb / sec / 1e9, "total_gbs": tb / sec / 1e9,
+                                "frac_of_peak_total": tb / sec / 1e9 / peak}
+            del gs
+        dense = sweep.get("1")
+        if dense:
+            for v in sweep.values():
+                v["speedup_vs_p1"] = v["tokens_per_s"] / dense["tokens_per_s"]
+
+    # ---- warm-L2 number (no flush), for context
+    warm = time_graphs(graphs, min(args.steps, 500), 5, None, stream)
+    warm_tok_s = B * len(warm) / (sum(warm) / 1e3)
+
+    # ---- end to end through the public API with host buffers
+    x_host = [torch.empty((B, w.d_model), dtype=layers[0]["x"].dtype, pin_memory=True) for _ in layers]
+    y_host = [torch.empty((B, w.d_model), dtype=layers[0]["x"].dtype, pin_memory=True) for _ in layers]
+    for l, L in enumerate(layers):
+        x_host[l].copy_(L["x"][0].cpu())
+    x_dev = [torch.empty_like(L["y"]) for L in layers]
+    e2e_steps = min(args.steps, 300)
+    with torch.cuda.stream(stream):
+        for rep in range(2):
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            for _ in range(e2e_steps if rep else 5):
+                for l, L in enumerate(layers):
+                    x_dev[l].copy_(x_host[l], non_blocking=True)
+                    pp.pp_layer(desc, x_dev[l], B, L["Wr"], L["Wg"], L["Wu"], L["Wd"], pf, None, L["y"], ws,
+                                stream=stream)
+                    y_host[l].copy_(L["y"], non_blocking=True)
+                stream.synchronize()
+            el = time.perf_counter() - t0
+    el_max = max_over_ranks(el)
+    e2e = {"value": world * B * e2e_steps / el_max,
+           "unit": "tokens/s", "h2d_bytes_per_step": w.n_layers * B * w.d_model * (2 if w.dtype == "bf16" else 4),
+           "d2h_bytes_per_step": w.n_layers * B * w.d_model * (2 if w.dtype == "bf16" else 4),
+           "path": "pp_layer via the ctypes binding, eager launches, pinned host x/y copied every layer"}
+
+    out = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+           "config": {"workload": w.name, "d_model": w.d_model, "d_ff": w.d_ff, "n_experts": w.n_experts,
+                      "d_expert": 64, "layers": w.n_layers, "batch": B, "p": args.p, "act": w.act,
+                      "token_pool": args.pool,
+                      "l2": "no flush (warm)" if args.no_flush else "flushed between steps (256 MiB write, untimed)",
+                      "parallelism": "replicas" if world > 1 else "single GPU"},
+           "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                        "frac": achieved / peak, "traffic": kernel_traffic(w.name, args.p),
+                        "peak_kind": peak_kind, "kernel": "decode_layer_kernel",
+                        "bytes_per_launch": bytes_per_launch, "launch_ms": per_launch_ms},
+           "expert_bytes": {"gbs": expert_gbs, "frac_of_peak": expert_gbs / peak,
+                            "frac_of_8tbs": expert_gbs / 8000.0, "k_mean": k_mean, "s_ffn": s_ffn},
+           "p_sweep": sweep, "warm_l2_tokens_per_s": warm_tok_s,
+           "e2e": e2e, "gpu_launches": launches, "clocks": clocks}
+    if rank == 0 and world == 1:
+        try:
+            out["cpu_baseline"] = run_oracle_sample(w, args.cpu_seconds, args.seed, p=args.p, B=B)
+        except Exception as ex:  # the oracle needs gcc; report rather than fail the bench
+            out["cpu_baseline"] = {"value": None, "error": str(ex)[:200]}
+    if rank == 0:
+        print(json.dumps(out))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

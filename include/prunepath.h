@@ -1,0 +1,168 @@
+/*
+ * prunepath.h -- C ABI of the GB300 (sm_103a) PrunePath sparse-FFN library.
+ *
+ * PrunePath (Sec. 3.1) routes each token x in R^d with a linear router
+ *   g = W_r^T x                                   (Eq. routing_logits)
+ *   p_j = exp(g_j) / sum_i exp(g_i)               (Eq. softmax_prob)
+ * orders the experts by descending probability (pi), activates a prefix of
+ * that order by cumulative probability mass     (Eq. tau_thresh_activate)
+ * and evaluates only the activated expert slices of a MoEfied FFN
+ *   y = sum_{e in A} sigmoid(g_e) * FFN_e(x)      (Eq. moe_output)
+ * where FFN_e is the restriction of the gated FFN (Eq. ffn) to the e-th block
+ * of d_e contiguous intermediate neurons        (Eq. moefication_decomp).
+ *
+ * ------------------------------------------------------------------------
+ * Conventions shared by every entry point
+ *  - Every tensor pointer is a DEVICE pointer owned by the caller, row-major,
+ *    contiguous and 16-byte aligned.  The library never allocates, frees or
+ *    keeps a tensor pointer beyond the call.
+ *  - Weight layout ("expert neurons stored contiguously"):
+ *      W_r    [E][d]      row j is the routing vector of expert j
+ *                         (the paper's W_r in R^{d x E}, stored transposed)
+ *      W_gate [d_ff][d]   row n holds neuron n's input weights; expert e is
+ *      W_up   [d_ff][d]   the dense row block [e*d_e, (e+1)*d_e)
+ *      W_down [d][d_ff]   expert e is the dense column block [e*d_e, (e+1)*d_e)
+ *    x and y are [T][d].  Element type: pp_desc.dtype for x, y and all weights.
+ *  - The selection (pp_selection) is [T][E] int32 ids in rank order (first
+ *    counts[t] entries valid, the rest -1), counts [T] int32, gates [T][E]
+ *    fp32 aligned with ids (sigmoid(g_e) for PP_GATE_SIGMOID, 1 for
+ *    PP_GATE_NONE, 0 past counts[t]) and, optionally, logits [T][E] fp32 in
+ *    expert order.
+ *  - Every call is asynchronous on `stream` (a cudaStream_t passed as void*;
+ *    NULL means the legacy default stream).  Argument errors are returned
+ *    synchronously before anything is enqueued.  Errors found on the device
+ *    (a bounded wait that timed out, a non-finite logit) are recorded in the
+ *    workspace status word and read back by pp_get_device_status.
+ *  - Workspace: caller-owned device memory of at least pp_workspace_size()
+ *    bytes, 256-byte aligned, zeroed once by pp_workspace_init before its
+ *    first use.  Calls that share a workspace must be ordered on one stream;
+ *    calls on different workspaces are independent.
+ *  - No C++ exception crosses this interface.
+ *  - Supported shapes: d_expert == 64, d_ff == E * 64, 1 <= E <= 256,
+ *    d a multiple of 8 (bf16) or 4 (fp32), 64 <= d <= 8192, T >= 0.
+ *    Other shapes return PP_ERR_SHAPE.
+ *  - p semantics: p >= 1 activates all E experts (the warm-up setting
+ *    tau_warm = 1.05 of Sec. 3.2); p <= 0 activates the top-1 expert only;
+ *    NaN returns PP_ERR_INVALID_ARG.
+ */
+#ifndef PRUNEPATH_H
+#define PRUNEPATH_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum pp_status {
+    PP_OK = 0,
+    PP_ERR_INVALID_ARG = 1, /* NULL pointer, NaN p, unknown enum value            */
+    PP_ERR_SHAPE = 2,       /* shape outside the supported set (see above)        */
+    PP_ERR_DTYPE = 3,       /* unsupported dtype / activation combination         */
+    PP_ERR_ALIGN = 4,       /* a pointer is not 16-byte aligned                   */
+    PP_ERR_WORKSPACE = 5,   /* workspace NULL, misaligned or too small            */
+    PP_ERR_CUDA = 6,        /* a CUDA runtime call failed (launch, attribute)     */
+    PP_ERR_TIMEOUT = 7,     /* device: a bounded wait gave up (sticky)            */
+    PP_ERR_CAPACITY = 8,    /* device: an internal buffer would overflow (sticky) */
+    PP_ERR_NONFINITE = 9,   /* device: a router logit was NaN/Inf (sticky); the
+                               token gets counts[t] = 0 and y[t] = 0              */
+    PP_ERR_UNSUPPORTED = 10 /* no device of compute capability 10.3 is current    */
+} pp_status;
+
+typedef enum pp_dtype { PP_F32 = 0, PP_BF16 = 1 } pp_dtype;
+
+/* FFN variant.  SWIGLU is Eq. (ffn) with phi = SiLU and needs W_gate; RELU
+   and GELU_TANH are the non-gated forms h = phi(x W_up) (Sec. 2.1 notes the
+   analysis covers any FFN separable along d_ff) and take W_gate = NULL. */
+typedef enum pp_act { PP_ACT_RELU = 0, PP_ACT_GELU_TANH = 1, PP_ACT_SWIGLU = 2 } pp_act;
+
+/* Output weighting.  SIGMOID is Eq. (moe_output); NONE weights every
+   selected expert by 1, the plain decomposition of Eq. (moefication_decomp). */
+typedef enum pp_gate { PP_GATE_SIGMOID = 0, PP_GATE_NONE = 1 } pp_gate;
+
+/* Cut rule on the descending order pi with inclusive prefix masses S_i.
+   MIN_PREFIX: the shortest prefix whose mass reaches p (keeps the rank that
+   crosses p).  PAPER: Eq. (tau_thresh_activate) literally, rank 1 plus every
+   rank with S_i < p.  Whenever S_E >= p, |PAPER| = max(1, |MIN_PREFIX| - 1). */
+typedef enum pp_rule { PP_SEL_MIN_PREFIX = 0, PP_SEL_PAPER = 1 } pp_rule;
+
+typedef struct pp_desc {
+    int d_model;   /* d                                   */
+    int d_ff;      /* intermediate width, == n_experts*64 */
+    int n_experts; /* E                                   */
+    int d_expert;  /* d_e, must be 64                     */
+    int dtype;     /* pp_dtype                            */
+    int act;       /* pp_act                              */
+    int gate;      /* pp_gate                             */
+    int rule;      /* pp_rule                             */
+} pp_desc;
+
+typedef struct pp_selection {
+    int32_t *ids;    /* [T][E] device, rank order, -1 padded          */
+    int32_t *counts; /* [T]    device                                 */
+    float *gates;    /* [T][E] device, aligned with ids               */
+    float *logits;   /* [T][E] device, expert order; may be NULL      */
+} pp_selection;
+
+/* Bytes of workspace needed for calls with up to T tokens. */
+size_t pp_workspace_size(const pp_desc *desc, int T);
+
+/* Zero the workspace's control words (status, barrier counters) on `stream`.
+   Call once after allocating a workspace, and again to clear a sticky
+   device error. */
+pp_status pp_workspace_init(void *ws, size_t ws_bytes, void *stream);
+
+/* Router and selection (Eq. routing_logits, softmax_prob,
+   tau_thresh_activate).  x [T][d], W_r [E][d]; writes *out (out->logits may
+   be NULL).  The softmax is max-shifted in fp32 with fp32 exponentials; the
+   normaliser and the prefix masses are accumulated in fp64; the order is
+   descending logit with ties broken by the lower expert index. */
+pp_status pp_route(const pp_desc *desc, const void *x, int T, const void *W_r, float p,
+                   const pp_selection *out, void *ws, size_t ws_bytes, void *stream);
+
+/* Selection only, from given fp32 logits [T][E] (out->logits is ignored). */
+pp_status pp_select(const pp_desc *desc, const float *logits, int T, float p,
+                    const pp_selection *out, void *ws, size_t ws_bytes, void *stream);
+
+/* Sparse FFN over a given selection (Eq. moe_output): for each token t,
+   y[t] = sum_{r < counts[t]} gates[t][r] * FFN_{ids[t][r]}(x[t]).
+   Reads sel->ids, sel->counts, sel->gates.  W_gate is NULL unless act is
+   PP_ACT_SWIGLU.  Accumulation is fp32; y has the dtype of x. */
+pp_status pp_sparse_ffn(const pp_desc *desc, const void *x, int T, const void *W_gate,
+                        const void *W_up, const void *W_down, const pp_selection *sel, void *y,
+                        void *ws, size_t ws_bytes, void *stream);
+
+/* pp_route followed by pp_sparse_ffn, fused where the token count allows.
+   sel_out may be NULL (the selection then stays in the workspace). */
+pp_status pp_layer(const pp_desc *desc, const void *x, int T, const void *W_r, const void *W_gate,
+                   const void *W_up, const void *W_down, float p, const pp_selection *sel_out,
+                   void *y, void *ws, size_t ws_bytes, void *stream);
+
+/* FFN-sparsity statistics (Sec. 4.1, s_FFN): adds sum_t counts[t] to
+   acc[0] and a histogram of counts (0..E) to acc[1..E+1].  acc is
+   [E+2] uint64 on the device, accumulated across calls (one per layer), so
+   s_FFN = 1 - acc[0] / (N * L * E). */
+pp_status pp_sparsity_stats(const int32_t *counts, int T, int n_experts, uint64_t *acc,
+                            void *stream);
+
+/* Synchronise `stream` and return the sticky device status of `ws`. */
+pp_status pp_get_device_status(void *ws, void *stream);
+
+/* Test hook for failure detection: enqueue one kernel that waits on a
+   workspace flag nothing sets, with a limit of timeout_ns nanoseconds; it
+   then records PP_ERR_TIMEOUT in the workspace status and returns.  No GPU
+   fault, trap or hang is involved. */
+pp_status pp_debug_wait_timeout(void *ws, size_t ws_bytes, long long timeout_ns, void *stream);
+
+/* Human-readable name of a status code (static string). */
+const char *pp_status_string(pp_status s);
+
+/* Library version, "major.minor.patch". */
+const char *pp_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PRUNEPATH_H */

@@ -1,0 +1,384 @@
+// C ABI of libprunepath: argument checks, workspace layout and dispatch to
+// the kernels.  Everything is enqueued on the caller's stream; nothing here
+// allocates device memory or synchronises (except pp_get_device_status).
+#include <cmath>
+#include <cstring>
+#include <mutex>
+
+#include <cudaTypedefs.h>
+
+#include "pp_common.cuh"
+#include "pp_kernels.h"
+
+namespace pp {
+namespace {
+
+constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;  // bounded waits give up after 2 s
+
+struct DeviceInfo {
+    int sms = 0, cc_major = 0, cc_minor = 0;
+    size_t smem_optin = 0;
+    bool ok = false;
+};
+
+DeviceInfo device_info() {
+    static std::mutex mu;
+    static DeviceInfo cache[64];
+    static bool have[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return DeviceInfo{};
+    std::lock_guard<std::mutex> lock(mu);
+    if (!have[dev]) {
+        DeviceInfo d;
+        int v = 0;
+        bool ok = cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess;
+        ok = ok && cudaDeviceGetAttribute(&d.cc_major, cudaDevAttrComputeCapabilityMajor, dev) == cudaSuccess;
+        ok = ok && cudaDeviceGetAttribute(&d.cc_minor, cudaDevAttrComputeCapabilityMinor, dev) == cudaSuccess;
+        ok = ok && cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) == cudaSuccess;
+        d.smem_optin = (size_t)v;
+        d.ok = ok;
+        cache[dev] = d;
+        have[dev] = true;
+    }
+    return cache[dev];
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
+
+// Workspace layout for calls with up to T tokens.
+struct Layout {
+    size_t logits, ids, counts, gates, h, total;
+};
+
+Layout layout(const pp_desc& d, int T) {
+    const size_t E = (size_t)d.n_experts, Tn = (size_t)(T > 0 ? T : 1);
+    Layout L{};
+    size_t off = sizeof(Control);
+    L.logits = off;
+    off = align256(off + Tn * E * 4);
+    L.ids = off;
+    off = align256(off + Tn * E * 4);
+    L.counts = off;
+    off = align256(off + Tn * 4);
+    L.gates = off;
+    off = align256(off + Tn * E * 4);
+    L.h = off;
+    off = align256(off + E * 8 * kDExpert * 4);
+    L.total = off;
+    return L;
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+pp_status check_desc(const pp_desc* d) {
+    if (!d) return PP_ERR_INVALID_ARG;
+    if (d->dtype != PP_F32 && d->dtype != PP_BF16) return PP_ERR_DTYPE;
+    if (d->act < PP_ACT_RELU || d->act > PP_ACT_SWIGLU) return PP_ERR_INVALID_ARG;
+    if (d->gate != PP_GATE_SIGMOID && d->gate != PP_GATE_NONE) return PP_ERR_INVALID_ARG;
+    if (d->rule != PP_SEL_MIN_PREFIX && d->rule != PP_SEL_PAPER) return PP_ERR_INVALID_ARG;
+    if (d->d_expert != kDExpert) return PP_ERR_SHAPE;
+    if (d->n_experts < 1 || d->n_experts > kMaxExperts) return PP_ERR_SHAPE;
+    if ((long long)d->d_ff != (long long)d->n_experts * kDExpert) return PP_ERR_SHAPE;
+    const int vec = d->dtype == PP_BF16 ? 8 : 4;
+    if (d->d_model < 64 || d->d_model > kMaxD || d->d_model % vec != 0) return PP_ERR_SHAPE;
+    return PP_OK;
+}
+
+pp_status check_T(const pp_desc* d, int T) {
+    if (T < 0) return PP_ERR_SHAPE;
+    if ((long long)T * d->n_experts > (1ll << 31) - 1 || (long long)T * d->d_model > (1ll << 31) - 1)
+        return PP_ERR_SHAPE;
+    return PP_OK;
+}
+
+pp_status check_ws(const pp_desc* d, int T, void* ws, size_t ws_bytes) {
+    if (!ws || ((uintptr_t)ws & 255u) != 0) return PP_ERR_WORKSPACE;
+    if (ws_bytes < layout(*d, T).total) return PP_ERR_WORKSPACE;
+    return PP_OK;
+}
+
+pp_status check_device() {
+    const DeviceInfo di = device_info();
+    if (!di.ok) return PP_ERR_CUDA;
+    if (di.cc_major != 10 || di.cc_minor != 3) return PP_ERR_UNSUPPORTED;
+    return PP_OK;
+}
+
+pp_status check_sel(const pp_selection* s) {
+    if (!s || !s->ids || !s->counts || !s->gates) return PP_ERR_INVALID_ARG;
+    if (!aligned16(s->ids) || !aligned16(s->counts) || !aligned16(s->gates)) return PP_ERR_ALIGN;
+    if (s->logits && !aligned16(s->logits)) return PP_ERR_ALIGN;
+    return PP_OK;
+}
+
+pp_status check_weights(const pp_desc* d, const void* Wg, const void* Wu, const void* Wd) {
+    if (!Wu || !Wd) return PP_ERR_INVALID_ARG;
+    if (d->act == PP_ACT_SWIGLU && !Wg) return PP_ERR_INVALID_ARG;
+    if (!aligned16(Wu) || !aligned16(Wd) || (d->act == PP_ACT_SWIGLU && !aligned16(Wg))) return PP_ERR_ALIGN;
+    return PP_OK;
+}
+
+pp_status cuda_status(cudaError_t e) { return e == cudaSuccess ? PP_OK : PP_ERR_CUDA; }
+
+#define PP_TRY(expr)                        \
+    do {                                    \
+        const pp_status _s = (expr);        \
+        if (_s != PP_OK) return _s;         \
+    } while (0)
+
+struct Ws {
+    Control* ctrl;
+    float* logits;
+    int32_t* ids;
+    int32_t* counts;
+    float* gates;
+    float* h;
+};
+
+Ws ws_views(const pp_desc& d, int T, void* ws) {
+    const Layout L = layout(d, T);
+    char* b = static_cast<char*>(ws);
+    return Ws{reinterpret_cast<Control*>(b), reinterpret_cast<float*>(b + L.logits),
+              reinterpret_cast<int32_t*>(b + L.ids), reinterpret_cast<int32_t*>(b + L.counts),
+              reinterpret_cast<float*>(b + L.gates), reinterpret_cast<float*>(b + L.h)};
+}
+
+bool make_down_map(const pp_desc& d, const void* Wd, int R6, CUtensorMap* map) {
+    auto enc = tensor_map_encoder();
+    if (!enc) return false;
+    const bool bf = d.dtype == PP_BF16;
+    const cuuint64_t dims[2] = {(cuuint64_t)d.d_ff, (cuuint64_t)d.d_model};
+    const cuuint64_t strides[1] = {(cuuint64_t)d.d_ff * (bf ? 2 : 4)};
+    const cuuint32_t box[2] = {(cuuint32_t)kDExpert, (cuuint32_t)R6};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult r = enc(map, bf ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2,
+                           const_cast<void*>(Wd), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                           CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+// One launch of the fused decode kernel over tokens [t0, t0 + n).
+pp_status decode_call(const pp_desc& d, const void* x, int t0, int n, const void* Wr, const void* Wg,
+                      const void* Wu, const void* Wd, float p, const pp_selection* sel, bool do_route,
+                      bool do_ffn, void* y, const Ws& w, cudaStream_t st) {
+    const DeviceInfo di = device_info();
+    int TS = 1;
+    while (TS < n) TS <<= 1;
+    if (TS > decode_max_ts(d.dtype)) return PP_ERR_SHAPE;
+    // leave 2 KB of the opt-in limit for the kernel's static shared memory
+    DecodePlanIn in{d.dtype, d.d_model, d.n_experts, TS, di.sms, d.act == PP_ACT_SWIGLU, di.smem_optin - 2048};
+    DecodePlan plan;
+    if (!decode_plan(in, &plan)) return PP_ERR_SHAPE;
+    DecodeArgs a;
+    std::memset(&a, 0, sizeof a);
+    const size_t esz = d.dtype == PP_BF16 ? 2 : 4;
+    if (do_ffn && !make_down_map(d, Wd, plan.R6, &a.tmap_down)) return PP_ERR_CUDA;
+    const size_t E = (size_t)d.n_experts;
+    a.x = static_cast<const char*>(x) + (size_t)t0 * d.d_model * esz;
+    a.Wr = Wr;
+    a.Wg = Wg;
+    a.Wu = Wu;
+    a.y = y ? static_cast<char*>(y) + (size_t)t0 * d.d_model * esz : nullptr;
+    if (sel) {
+        a.sel_ids = sel->ids + (size_t)t0 * E;
+        a.sel_counts = sel->counts + t0;
+        a.sel_gates = sel->gates + (size_t)t0 * E;
+        a.sel_logits = sel->logits ? sel->logits + (size_t)t0 * E : nullptr;
+    }
+    a.logit_ws = w.logits;
+    a.h_ws = w.h;
+    a.status = &w.ctrl->status;
+    a.bar = &w.ctrl->grid_bar[0];
+    a.timeout_ns = kDefaultTimeoutNs;
+    a.T = n;
+    a.d = d.d_model;
+    a.E = d.n_experts;
+    a.act = d.act;
+    a.gate = d.gate;
+    a.rule = d.rule;
+    a.p = p;
+    a.do_route = do_route ? 1 : 0;
+    a.do_ffn = do_ffn ? 1 : 0;
+    a.sel_slots = sel_slots_for(d.n_experts);
+    a.R6 = plan.R6;
+    a.NS4 = plan.NS4;
+    a.uch = plan.uch;
+    a.off_x = plan.off_x;
+    a.off_gw = plan.off_gw;
+    a.off_mask = plan.off_mask;
+    a.off_ulist = plan.off_ulist;
+    a.off_red = plan.off_red;
+    a.off_h = plan.off_h;
+    a.off_ring6 = plan.off_ring6;
+    a.off_ring4 = plan.off_ring4;
+    return cuda_status(decode_launch(a, plan, d.dtype, TS, di.sms, st));
+}
+
+}  // namespace
+}  // namespace pp
+
+using namespace pp;
+
+extern "C" {
+
+size_t pp_workspace_size(const pp_desc* desc, int T) {
+    if (check_desc(desc) != PP_OK || T < 0) return 0;
+    return layout(*desc, T).total;
+}
+
+pp_status pp_workspace_init(void* ws, size_t ws_bytes, void* stream) {
+    if (!ws || ((uintptr_t)ws & 255u) != 0 || ws_bytes < sizeof(Control)) return PP_ERR_WORKSPACE;
+    return cuda_status(cudaMemsetAsync(ws, 0, sizeof(Control), static_cast<cudaStream_t>(stream)));
+}
+
+pp_status pp_select(const pp_desc* desc, const float* logits, int T, float p, const pp_selection* out,
+                    void* ws, size_t ws_bytes, void* stream) {
+    PP_TRY(check_desc(desc));
+    PP_TRY(check_T(desc, T));
+    if (std::isnan(p)) return PP_ERR_INVALID_ARG;
+    PP_TRY(check_sel(out));
+    if (!logits) return PP_ERR_INVALID_ARG;
+    if (!aligned16(logits)) return PP_ERR_ALIGN;
+    PP_TRY(check_ws(desc, T, ws, ws_bytes));
+    PP_TRY(check_device());
+    if (T == 0) return PP_OK;
+    const Ws w = ws_views(*desc, T, ws);
+    return cuda_status(select_launch(logits, T, desc->n_experts, p, desc->rule, desc->gate, out->ids,
+                                     out->counts, out->gates, &w.ctrl->status,
+                                     static_cast<cudaStream_t>(stream)));
+}
+
+pp_status pp_route(const pp_desc* desc, const void* x, int T, const void* W_r, float p,
+                   const pp_selection* out, void* ws, size_t ws_bytes, void* stream) {
+    PP_TRY(check_desc(desc));
+    PP_TRY(check_T(desc, T));
+    if (std::isnan(p)) return PP_ERR_INVALID_ARG;
+    PP_TRY(check_sel(out));
+    if (!x || !W_r) return PP_ERR_INVALID_ARG;
+    if (!aligned16(x) || !aligned16(W_r)) return PP_ERR_ALIGN;
+    PP_TRY(check_ws(desc, T, ws, ws_bytes));
+    PP_TRY(check_device());
+    if (T == 0) return PP_OK;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const Ws w = ws_views(*desc, T, ws);
+    if (T <= decode_max_ts(desc->dtype))
+        return decode_call(*desc, x, 0, T, W_r, nullptr, nullptr, nullptr, p, out, true, false, nullptr, w, st);
+    float* lg = out->logits ? out->logits : w.logits;
+    PP_TRY(cuda_status(router_launch(desc->dtype, x, T, desc->d_model, W_r, desc->n_experts, lg, st)));
+    return cuda_status(select_launch(lg, T, desc->n_experts, p, desc->rule, desc->gate, out->ids, out->counts,
+                                     out->gates, &w.ctrl->status, st));
+}
+
+pp_status pp_sparse_ffn(const pp_desc* desc, const void* x, int T, const void* W_gate, const void* W_up,
+                        const void* W_down, const pp_selection* sel, void* y, void* ws, size_t ws_bytes,
+                        void* stream) {
+    PP_TRY(check_desc(desc));
+    PP_TRY(check_T(desc, T));
+    PP_TRY(check_sel(sel));
+    if (!x || !y) return PP_ERR_INVALID_ARG;
+    if (!aligned16(x) || !aligned16(y)) return PP_ERR_ALIGN;
+    PP_TRY(check_weights(desc, W_gate, W_up, W_down));
+    PP_TRY(check_ws(desc, T, ws, ws_bytes));
+    PP_TRY(check_device());
+    if (T == 0) return PP_OK;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const Ws w = ws_views(*desc, T, ws);
+    const int ts = decode_max_ts(desc->dtype);
+    for (int t0 = 0; t0 < T; t0 += ts) {
+        const int n = std::min(ts, T - t0);
+        PP_TRY(decode_call(*desc, x, t0, n, nullptr, W_gate, W_up, W_down, 0.0f, sel, false, true, y, w, st));
+    }
+    return PP_OK;
+}
+
+pp_status pp_layer(const pp_desc* desc, const void* x, int T, const void* W_r, const void* W_gate,
+                   const void* W_up, const void* W_down, float p, const pp_selection* sel_out, void* y,
+                   void* ws, size_t ws_bytes, void* stream) {
+    PP_TRY(check_desc(desc));
+    PP_TRY(check_T(desc, T));
+    if (std::isnan(p)) return PP_ERR_INVALID_ARG;
+    if (sel_out) PP_TRY(check_sel(sel_out));
+    if (!x || !y || !W_r) return PP_ERR_INVALID_ARG;
+    if (!aligned16(x) || !aligned16(y) || !aligned16(W_r)) return PP_ERR_ALIGN;
+    PP_TRY(check_weights(desc, W_gate, W_up, W_down));
+    PP_TRY(check_ws(desc, T, ws, ws_bytes));
+    PP_TRY(check_device());
+    if (T == 0) return PP_OK;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const Ws w = ws_views(*desc, T, ws);
+    if (T <= decode_max_ts(desc->dtype))
+        return decode_call(*desc, x, 0, T, W_r, W_gate, W_up, W_down, p, sel_out, true, true, y, w, st);
+    pp_selection s = sel_out ? *sel_out : pp_selection{w.ids, w.counts, w.gates, nullptr};
+    float* lg = s.logits ? s.logits : w.logits;
+    PP_TRY(cuda_status(router_launch(desc->dtype, x, T, desc->d_model, W_r, desc->n_experts, lg, st)));
+    PP_TRY(cuda_status(select_launch(lg, T, desc->n_experts, p, desc->rule, desc->gate, s.ids, s.counts, s.gates,
+                                     &w.ctrl->status, st)));
+    const int ts = decode_max_ts(desc->dtype);
+    for (int t0 = 0; t0 < T; t0 += ts) {
+        const int n = std::min(ts, T - t0);
+        PP_TRY(decode_call(*desc, x, t0, n, nullptr, W_gate, W_up, W_down, 0.0f, &s, false, true, y, w, st));
+    }
+    return PP_OK;
+}
+
+pp_status pp_sparsity_stats(const int32_t* counts, int T, int n_experts, uint64_t* acc, void* stream) {
+    if (!counts || !acc || T < 0 || n_experts < 1 || n_experts > kMaxExperts) return PP_ERR_INVALID_ARG;
+    if (((uintptr_t)counts & 3u) || ((uintptr_t)acc & 7u)) return PP_ERR_ALIGN;
+    PP_TRY(check_device());
+    return cuda_status(stats_launch(counts, T, n_experts, acc, static_cast<cudaStream_t>(stream)));
+}
+
+pp_status pp_get_device_status(void* ws, void* stream) {
+    if (!ws || ((uintptr_t)ws & 255u) != 0) return PP_ERR_WORKSPACE;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    unsigned v = 0;
+    if (cudaMemcpyAsync(&v, &static_cast<Control*>(ws)->status, sizeof v, cudaMemcpyDeviceToHost, st) !=
+        cudaSuccess)
+        return PP_ERR_CUDA;
+    if (cudaStreamSynchronize(st) != cudaSuccess) return PP_ERR_CUDA;
+    return static_cast<pp_status>(v);
+}
+
+pp_status pp_debug_wait_timeout(void* ws, size_t ws_bytes, long long timeout_ns, void* stream) {
+    if (!ws || ((uintptr_t)ws & 255u) != 0 || ws_bytes < sizeof(Control)) return PP_ERR_WORKSPACE;
+    if (timeout_ns <= 0 || timeout_ns > 10000000000ll) return PP_ERR_INVALID_ARG;
+    PP_TRY(check_device());
+    Control* c = static_cast<Control*>(ws);
+    return cuda_status(wait_timeout_launch(&c->wait_flag, &c->status, timeout_ns, static_cast<cudaStream_t>(stream)));
+}
+
+const char* pp_status_string(pp_status s) {
+    switch (s) {
+        case PP_OK: return "PP_OK";
+        case PP_ERR_INVALID_ARG: return "PP_ERR_INVALID_ARG";
+        case PP_ERR_SHAPE: return "PP_ERR_SHAPE";
+        case PP_ERR_DTYPE: return "PP_ERR_DTYPE";
+        case PP_ERR_ALIGN: return "PP_ERR_ALIGN";
+        case PP_ERR_WORKSPACE: return "PP_ERR_WORKSPACE";
+        case PP_ERR_CUDA: return "PP_ERR_CUDA";
+        case PP_ERR_TIMEOUT: return "PP_ERR_TIMEOUT";
+        case PP_ERR_CAPACITY: return "PP_ERR_CAPACITY";
+        case PP_ERR_NONFINITE: return "PP_ERR_NONFINITE";
+        case PP_ERR_UNSUPPORTED: return "PP_ERR_UNSUPPORTED";
+    }
+    return "PP_ERR_UNKNOWN";
+}
+
+const char* pp_version(void) { return "0.1.0"; }
+
+}  // extern "C"

@@ -1,0 +1,207 @@
+// Device helpers shared by the PrunePath kernels (sm_103a).
+//
+// Inline PTX wrappers for mbarriers, bulk and tensor TMA copies, proxy
+// fences and the global timer; a bounded mbarrier wait; a self-resetting
+// grid barrier for cooperative (co-resident) grids; bf16 helpers.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "prunepath.h"
+
+#define PP_DEVINL __device__ __forceinline__
+
+namespace pp {
+
+constexpr int kDExpert = 64;      // d_e, the expert width this library is built for
+constexpr int kMaxExperts = 256;  // E limit (the warp sort holds 8 keys per lane)
+constexpr int kMaxD = 8192;
+constexpr unsigned kFull = 0xffffffffu;
+
+// ------------------------------------------------------------------ control
+// The first 256 bytes of every workspace.
+struct Control {
+    unsigned status;      // sticky pp_status of the device side
+    unsigned wait_flag;   // never written: target of pp_debug_wait_timeout
+    unsigned grid_bar[4]; // self-resetting grid barrier counters
+    unsigned pad[58];
+};
+static_assert(sizeof(Control) == 256, "control block is 256 bytes");
+
+PP_DEVINL void record_status(unsigned* status, pp_status s) {
+    // first error wins; later ones do not overwrite it
+    atomicCAS(status, 0u, (unsigned)s);
+}
+
+PP_DEVINL uint64_t globaltimer_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// ----------------------------------------------------------------- mbarrier
+PP_DEVINL uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+PP_DEVINL void mbar_init(uint64_t* bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+
+PP_DEVINL void fence_mbar_init() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
+
+PP_DEVINL void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+                 "r"(bytes)
+                 : "memory");
+}
+
+PP_DEVINL void mbar_arrive(uint64_t* bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+PP_DEVINL bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait for the phase with the given parity to complete, for at most
+// limit_ns.  On expiry records PP_ERR_TIMEOUT and returns false.
+PP_DEVINL bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned* status, uint64_t limit_ns) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    while (true) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (globaltimer_ns() - t0 > limit_ns) {
+            record_status(status, PP_ERR_TIMEOUT);
+            return false;
+        }
+    }
+}
+
+// -------------------------------------------------------------------- TMA
+// 1-D bulk copy global -> shared, completion counted in bytes on `bar`.
+// src, dst 16-byte aligned, bytes a multiple of 16.
+PP_DEVINL void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            smem_u32(dst)),
+        "l"(src), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// 2-D tiled tensor copy global -> shared.  c0 is the inner (contiguous)
+// coordinate; c0 * element size must be a multiple of 16 bytes.
+PP_DEVINL void tma_load_2d(void* dst, const CUtensorMap* map, int c0, int c1, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, "
+        "{%2, %3}], [%4];" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// Order this thread's earlier generic-proxy shared-memory accesses before
+// later async-proxy (TMA) accesses of the same memory.
+PP_DEVINL void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+PP_DEVINL void named_bar_sync(int id, int nthreads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// ------------------------------------------------------------ grid barrier
+PP_DEVINL unsigned ld_acquire_gpu(const unsigned* p) {
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Barrier across all CTAs of a co-resident (cooperative) grid.  The counter
+// returns to its starting value after every complete barrier, so one zeroed
+// word serves any number of barriers and launches.  Every thread of every
+// CTA must call it.  Bounded: after limit_ns the waiting CTA records
+// PP_ERR_TIMEOUT and continues.
+PP_DEVINL void grid_barrier(unsigned* counter, unsigned* status, uint64_t limit_ns) {
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const unsigned nblocks = gridDim.x * gridDim.y * gridDim.z;
+        const bool first = (blockIdx.x | blockIdx.y | blockIdx.z) == 0;
+        const unsigned add = first ? (0x80000000u - (nblocks - 1u)) : 1u;
+        __threadfence();
+        const unsigned old = atomicAdd(counter, add);
+        const uint64_t t0 = globaltimer_ns();
+        while (((ld_acquire_gpu(counter) ^ old) & 0x80000000u) == 0u) {
+            if (globaltimer_ns() - t0 > limit_ns) {
+                record_status(status, PP_ERR_TIMEOUT);
+                break;
+            }
+        }
+        __threadfence();
+    }
+    __syncthreads();
+}
+
+// ------------------------------------------------------------------- bf16
+PP_DEVINL float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
+PP_DEVINL float bf16hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+// Element access for the two storage types.
+template <typename TW>
+struct Elem;
+
+template <>
+struct Elem<float> {
+    static constexpr int kPer16B = 4;
+    PP_DEVINL static void unpack(const uint4& v, float* f) {
+        f[0] = __uint_as_float(v.x);
+        f[1] = __uint_as_float(v.y);
+        f[2] = __uint_as_float(v.z);
+        f[3] = __uint_as_float(v.w);
+    }
+    PP_DEVINL static void store(void* base, size_t i, float v) { reinterpret_cast<float*>(base)[i] = v; }
+};
+
+template <>
+struct Elem<__nv_bfloat16> {
+    static constexpr int kPer16B = 8;
+    PP_DEVINL static void unpack(const uint4& v, float* f) {
+        f[0] = bf16lo(v.x);
+        f[1] = bf16hi(v.x);
+        f[2] = bf16lo(v.y);
+        f[3] = bf16hi(v.y);
+        f[4] = bf16lo(v.z);
+        f[5] = bf16hi(v.z);
+        f[6] = bf16lo(v.w);
+        f[7] = bf16hi(v.w);
+    }
+    PP_DEVINL static void store(void* base, size_t i, float v) {
+        reinterpret_cast<__nv_bfloat16*>(base)[i] = __float2bfloat16_rn(v);
+    }
+};
+
+// ------------------------------------------------------------ activations
+PP_DEVINL float sigmoidf_(float v) { return 1.0f / (1.0f + expf(-v)); }
+
+// h for one neuron: a = x.W_up row, b = x.W_gate row (Eq. ffn; SiLU gate for
+// PP_ACT_SWIGLU, h = relu(a) or the tanh form of GELU otherwise).
+PP_DEVINL float act_h(int act, float a, float b) {
+    if (act == PP_ACT_SWIGLU) return b / (1.0f + expf(-b)) * a;
+    if (act == PP_ACT_RELU) return fmaxf(a, 0.0f);
+    const float k0 = 0.7978845608028654f;  // sqrt(2/pi)
+    return 0.5f * a * (1.0f + tanhf(k0 * (a + 0.044715f * a * a * a)));
+}
+
+PP_DEVINL float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+    return v;
+}
+
+}  // namespace pp

@@ -1,0 +1,297 @@
+"""GPU parity: the CUDA library (through its C ABI) against the CPU oracle.
+
+Cases cover all five workload shapes (tiny ReLU fp32, GPT-2-medium GELU,
+Llama-2-7B / Llama-3-8B SwiGLU decode, Llama-2-13B SwiGLU), both cut rules,
+both gate modes, p from <= 0 to >= 1, token counts that exercise the fused
+decode kernel (T <= 4 bf16 / 8 fp32), its token slices and the stand-alone
+router + selection kernels, plus the degenerate inputs (ties, signed zeros,
+huge and non-finite logits, T = 0).
+"""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2605_28283_gb300 import workloads as wl
+from parity import (BOUNDARY, Y_TOL, check_route_selection, check_select_exact, check_y, f32,
+                    layer_inputs, logit_tolerance, to_host, widen)
+
+pytestmark = pytest.mark.gpu
+
+
+def dev(a):
+    return wl.to_torch(a, "cuda")
+
+
+def run_layer(pp, w, L, p, rule="min_prefix", gate="sigmoid", T=None):
+    import torch
+    T = L.x.shape[0] if T is None else T
+    desc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act, gate, rule)
+    ws = pp.alloc_workspace(desc, T)
+    x, Wr, Wu, Wd = dev(L.x), dev(L.Wr), dev(L.Wu), dev(L.Wd)
+    Wg = None if L.Wg is None else dev(L.Wg)
+    sel = pp.Selection.empty(T, w.n_experts, "cuda")
+    y = torch.empty_like(x)
+    pp.pp_layer(desc, x, T, Wr, Wg, Wu, Wd, p, sel, y, ws)
+    torch.cuda.synchronize()
+    status = pp.pp_get_device_status(ws)
+    return (to_host(sel.counts), to_host(sel.ids), to_host(sel.logits), to_host(y), status)
+
+
+def layer_parity(pp, name, T, p, rule="min_prefix", gate="sigmoid", d=None, E=None, seed=0, layer=0):
+    w, L = layer_inputs(name, T, seed, layer, d, E)
+    pf = f32(p)
+    counts, ids, logits, y, status = run_layer(pp, w, L, pf, rule, gate)
+    assert status == pp.PP_OK, pp.status_name(status)
+    g_ref = oracle.logits(L.x, L.Wr)
+    tol_g = logit_tolerance(L.x, L.Wr)
+    assert np.all(np.abs(logits - g_ref) <= tol_g), "router logits"
+    eps = np.abs(logits - g_ref).max(axis=1)
+    unique, n_nonunique = check_route_selection(counts, ids, g_ref, eps, pf, rule)
+    ro_counts, ro_ids, _, _ = oracle.select(g_ref, pf, rule)
+    err = check_y(L, y, ro_counts, ro_ids, g_ref, w.n_experts, w.act, gate, Y_TOL[w.dtype], unique, counts, ids)
+    return err, n_nonunique
+
+
+# ------------------------------------------------------------------ pp_layer
+@pytest.mark.parametrize("p", [0.5, 0.9, 1.0])
+@pytest.mark.parametrize("T", [1, 3, 8, 64])
+def test_layer_tiny_relu_f32(pp, T, p):
+    layer_parity(pp, "tiny_relu_f32", T, p)
+
+
+@pytest.mark.parametrize("p", [0.5, 0.7, 0.9])
+@pytest.mark.parametrize("T", [1, 4, 16])
+def test_layer_gpt2m_gelu(pp, T, p):
+    layer_parity(pp, "gpt2m_gelu_bf16", T, p)
+
+
+@pytest.mark.parametrize("p", [0.3, 0.5, 0.7, 0.9, 1.0])
+def test_layer_llama2_7b_decode(pp, p):
+    layer_parity(pp, "llama2_7b_decode", 1, p)
+
+
+@pytest.mark.parametrize("T,p", [(1, 0.3), (1, 0.95), (2, 0.7), (8, 0.5), (8, 0.9)])
+def test_layer_llama3_8b(pp, T, p):
+    layer_parity(pp, "llama3_8b_batched", T, p)
+
+
+@pytest.mark.parametrize("T", [1, 4, 37])
+def test_layer_llama2_13b(pp, T):
+    layer_parity(pp, "llama2_13b_prefill", T, 0.7)
+
+
+@pytest.mark.parametrize("rule", ["min_prefix", "paper"])
+@pytest.mark.parametrize("gate", ["sigmoid", "none"])
+@pytest.mark.parametrize("p", [-0.5, 0.0, 0.4, 0.99, 1.0, 1.5])
+def test_layer_rules_gates(pp, rule, gate, p):
+    layer_parity(pp, "llama2_7b_decode", 3, p, rule, gate, d=512, E=40)
+
+
+@pytest.mark.parametrize("d,E,T", [(64, 1, 2), (128, 3, 5), (200, 33, 4), (2048, 256, 3), (8192, 100, 1)])
+def test_layer_odd_shapes(pp, d, E, T):
+    layer_parity(pp, "llama3_8b_batched", T, 0.8, d=d, E=E)
+
+
+def test_layer_dense_identity(pp):
+    """p >= 1 with unit gates is the dense FFN (Eq. moefication_decomp)."""
+    w, L = layer_inputs("gpt2m_gelu_bf16", 4)
+    counts, ids, logits, y, status = run_layer(pp, w, L, 1.0, gate="none")
+    assert np.all(counts == w.n_experts)
+    ref = oracle.dense_ffn(L.x, L.Wg, L.Wu, L.Wd, w.act)
+    err = np.abs(y - ref).max(axis=1) / np.abs(ref).max(axis=1)
+    assert err.max() <= Y_TOL["bf16"]
+
+
+# ---------------------------------------------------------- pp_sparse_ffn
+@pytest.mark.parametrize("name,T", [("tiny_relu_f32", 64), ("gpt2m_gelu_bf16", 16),
+                                    ("llama2_7b_decode", 1), ("llama3_8b_batched", 8),
+                                    ("llama2_13b_prefill", 5)])
+def test_sparse_ffn_given_selection(pp, name, T):
+    """Selection made by the oracle, FFN on the GPU."""
+    import torch
+    w, L = layer_inputs(name, T)
+    g = oracle.logits(L.x, L.Wr)
+    counts, ids, _, _ = oracle.select(g, 0.7, "min_prefix")
+    gates = np.zeros(ids.shape, np.float32)
+    for t in range(T):
+        for r in range(counts[t]):
+            gates[t, r] = 1.0 / (1.0 + np.exp(-g[t, ids[t, r]]))
+    desc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act)
+    ws = pp.alloc_workspace(desc, T)
+    sel = pp.Selection(dev(ids), dev(counts), dev(gates))
+    x = dev(L.x)
+    y = torch.empty_like(x)
+    pp.pp_sparse_ffn(desc, x, T, None if L.Wg is None else dev(L.Wg), dev(L.Wu), dev(L.Wd), sel, y, ws)
+    torch.cuda.synchronize()
+    assert pp.pp_get_device_status(ws) == pp.PP_OK
+    ref = oracle.sparse_ffn(L.x, L.Wg, L.Wu, L.Wd, counts, ids, g, w.n_experts, w.act, "sigmoid")
+    err = np.abs(to_host(y) - ref).max(axis=1) / np.abs(ref).max(axis=1)
+    assert err.max() <= Y_TOL[w.dtype]
+
+
+# ---------------------------------------------------------------- pp_route
+@pytest.mark.parametrize("name,T", [("tiny_relu_f32", 64), ("gpt2m_gelu_bf16", 4),
+                                    ("llama2_7b_decode", 1), ("llama3_8b_batched", 64),
+                                    ("llama2_13b_prefill", 300)])
+@pytest.mark.parametrize("rule", ["min_prefix", "paper"])
+def test_route(pp, name, T, rule):
+    import torch
+    w, L = layer_inputs(name, T)
+    desc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act, "sigmoid", rule)
+    ws = pp.alloc_workspace(desc, T)
+    sel = pp.Selection.empty(T, w.n_experts, "cuda")
+    p = f32(0.7)
+    pp.pp_route(desc, dev(L.x), T, dev(L.Wr), p, sel, ws)
+    torch.cuda.synchronize()
+    assert pp.pp_get_device_status(ws) == pp.PP_OK
+    g_ref = oracle.logits(L.x, L.Wr)
+    lg = to_host(sel.logits)
+    assert np.all(np.abs(lg - g_ref) <= logit_tolerance(L.x, L.Wr))
+    eps = np.abs(lg - g_ref).max(axis=1)
+    counts, ids = to_host(sel.counts), to_host(sel.ids)
+    check_route_selection(counts, ids, g_ref, eps, p, rule)
+    gates = to_host(sel.gates)
+    for t in range(T):
+        k = counts[t]
+        np.testing.assert_allclose(gates[t, :k], 1.0 / (1.0 + np.exp(-g_ref[t, ids[t, :k]])), rtol=1e-5, atol=1e-7)
+        assert np.all(gates[t, k:] == 0)
+
+
+# --------------------------------------------------------------- pp_select
+def select_gpu(pp, logits, p, rule, gate="sigmoid"):
+    import torch
+    T, E = logits.shape
+    desc = pp.make_desc(64, E, "bf16", "swiglu", gate, rule)
+    ws = pp.alloc_workspace(desc, T)
+    sel = pp.Selection.empty(T, E, "cuda", with_logits=False)
+    pp.pp_select(desc, dev(logits.astype(np.float32)), T, p, sel, ws)
+    torch.cuda.synchronize()
+    return to_host(sel.counts), to_host(sel.ids), to_host(sel.gates), pp.pp_get_device_status(ws)
+
+
+@pytest.mark.parametrize("E", [1, 5, 16, 33, 64, 100, 172, 216, 224, 256])
+@pytest.mark.parametrize("rule", ["min_prefix", "paper"])
+def test_select_bit_exact(pp, E, rule):
+    T = 2000
+    logits = wl.host_logits(T, E, std=3.0, seed=E)
+    total_boundary = 0
+    for p in (0.0, 0.3, 0.5, 0.7, 0.9, 0.95, 1.0):
+        pf = f32(p)
+        counts, ids, gates, status = select_gpu(pp, logits, pf, rule)
+        assert status == pp.PP_OK
+        g = logits.astype(np.float64)
+        total_boundary += check_select_exact(counts, ids, g, pf, rule)
+        for t in range(0, T, 97):
+            k = counts[t]
+            ref = 1.0 / (1.0 + np.exp(-g[t, ids[t, :k]]))
+            np.testing.assert_allclose(gates[t, :k], ref, rtol=2e-6, atol=1e-30)
+            assert np.all(gates[t, k:] == 0)
+    assert total_boundary <= T * 7 * 0.01
+
+
+def test_select_ties_and_zeros(pp):
+    rng = np.random.default_rng(5)
+    T, E = 500, 172
+    logits = (np.round(rng.standard_normal((T, E)) * 4) / 2).astype(np.float32)  # many exact ties
+    logits[0, :] = 0.0
+    logits[1, ::2] = -0.0
+    logits[2, :] = np.float32(-1e4)
+    logits[2, 7] = np.float32(1e4)
+    logits[3, :] = np.linspace(30, -30, E).astype(np.float32)
+    for rule in ("min_prefix", "paper"):
+        for gate in ("sigmoid", "none"):
+            for p in (0.1, 0.5, 0.75, 0.999, 1.0):
+                pf = f32(p)
+                counts, ids, gates, status = select_gpu(pp, logits, pf, rule, gate)
+                assert status == pp.PP_OK
+                check_select_exact(counts, ids, logits.astype(np.float64), pf, rule)
+                if gate == "none":
+                    for t in range(T):
+                        assert np.all(gates[t, :counts[t]] == 1.0)
+
+
+def test_select_nonfinite(pp):
+    logits = wl.host_logits(6, 40)
+    logits[1, 3] = np.nan
+    logits[4, 0] = np.inf
+    logits[5, 9] = -np.inf
+    counts, ids, gates, status = select_gpu(pp, logits, 0.5, "min_prefix")
+    assert status == pp.PP_ERR_NONFINITE
+    assert counts[1] == 0 and counts[4] == 0 and counts[5] == 0
+    assert np.all(ids[1] == -1) and np.all(gates[4] == 0)
+    ok = [0, 2, 3]
+    check_select_exact(counts[ok], ids[ok], logits[ok].astype(np.float64), 0.5, "min_prefix")
+
+
+def test_empty_inputs(pp):
+    import torch
+    desc = pp.make_desc(256, 16, "f32", "relu")
+    ws = pp.alloc_workspace(desc, 0)
+    x = torch.empty((0, 256), device="cuda")
+    w = torch.empty((16, 256), device="cuda")
+    wu = torch.empty((1024, 256), device="cuda")
+    wd = torch.empty((256, 1024), device="cuda")
+    sel = pp.Selection.empty(1, 16, "cuda")
+    y = torch.empty((1, 256), device="cuda")
+    pp.pp_layer(desc, y, 0, w, None, wu, wd, 0.5, sel, y, ws)
+    pp.pp_route(desc, y, 0, w, 0.5, sel, ws)
+    pp.pp_select(desc, sel.logits, 0, 0.5, sel, ws)
+    pp.pp_sparse_ffn(desc, y, 0, None, wu, wd, sel, y, ws)
+    assert pp.pp_get_device_status(ws) == pp.PP_OK
+
+
+# -------------------------------------------------------------- auxiliaries
+def test_sparsity_stats(pp):
+    import torch
+    rng = np.random.default_rng(3)
+    counts = rng.integers(1, 173, size=5000).astype(np.int32)
+    acc = torch.zeros(174, dtype=torch.int64, device="cuda")
+    for _ in range(3):  # accumulates across calls (one per layer)
+        pp.pp_sparsity_stats(dev(counts), len(counts), 172, acc)
+    a = to_host(acc)
+    assert a[0] == 3 * counts.sum()
+    np.testing.assert_array_equal(a[1:], 3 * np.bincount(counts, minlength=173))
+
+
+def test_bounded_wait_times_out(pp):
+    """Failure detection: a wait on a flag nothing sets gives up and reports."""
+    import torch
+    desc = pp.make_desc(256, 16, "f32", "relu")
+    ws = pp.alloc_workspace(desc, 1)
+    pp.pp_debug_wait_timeout(ws, 2_000_000)
+    assert pp.pp_get_device_status(ws) == pp.PP_ERR_TIMEOUT
+    pp.pp_workspace_init(ws)
+    assert pp.pp_get_device_status(ws) == pp.PP_OK
+    # the context is still usable
+    layer_parity(pp, "tiny_relu_f32", 3, 0.5)
+
+
+def test_graph_capture_matches_eager(pp):
+    import torch
+    w, L = layer_inputs("llama2_7b_decode", 1, d=1024, E=64)
+    desc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act)
+    ws = pp.alloc_workspace(desc, 1)
+    x, Wr, Wg, Wu, Wd = (dev(a) for a in (L.x, L.Wr, L.Wg, L.Wu, L.Wd))
+    y0 = torch.empty_like(x)
+    y1 = torch.empty_like(x)
+    pp.pp_layer(desc, x, 1, Wr, Wg, Wu, Wd, 0.7, None, y0, ws)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(g, stream=s):
+            pp.pp_layer(desc, x, 1, Wr, Wg, Wu, Wd, 0.7, None, y1, ws, stream=s)
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(y0, y1)
+    assert pp.pp_get_device_status(ws) == pp.PP_OK
+
+
+def test_deterministic(pp):
+    import torch
+    w, L = layer_inputs("llama3_8b_batched", 8)
+    a = run_layer(pp, w, L, 0.7)
+    b = run_layer(pp, w, L, 0.7)
+    for u, v in zip(a, b):
+        assert np.array_equal(np.asarray(u), np.asarray(v))
