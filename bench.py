@@ -46,6 +46,9 @@ def parse():
     ap.add_argument("--no-flush", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling runs)")
+    ap.add_argument("--skip-extras", action="store_true",
+                    help="only the headline timing (no warm/e2e/CPU legs); for profiler runs")
     return ap.parse_args()
 
 
@@ -303,6 +306,9 @@ def main():
     from paper_2605_28283_gb300 import workloads as wl
     pp.load()
     w = wl.WORKLOADS[args.workload]
+    if args.layers:
+        from dataclasses import replace
+        w = replace(w, n_layers=args.layers)
     B = args.batch
     desc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act)
     stream = torch.cuda.Stream()
@@ -382,6 +388,13 @@ def main():
         if dense:
             for v in sweep.values():
                 v["speedup_vs_p1"] = v["tokens_per_s"] / dense["tokens_per_s"]
+
+    if args.skip_extras:
+        if rank == 0:
+            print(json.dumps({"metric": METRIC, "value": value, "unit": "tokens/s", "ms_per_step": ms_per_step,
+                              "workload": w.name, "layers": w.n_layers, "p": args.p,
+                              "launch_ms": per_launch_ms, "bytes_per_launch": bytes_per_launch}))
+        return
 
     # ---- warm-L2 number (no flush), for context
     warm = time_graphs(graphs, min(args.steps, 500), 5, None, stream)

@@ -172,6 +172,22 @@ bool make_down_map(const pp_desc& d, const void* Wd, int R6, CUtensorMap* map) {
     return r == CUDA_SUCCESS;
 }
 
+DecodePlanIn plan_in(const pp_desc& d, int TS) {
+    const DeviceInfo di = device_info();
+    // leave 4 KB of the opt-in limit for the kernel's static shared memory
+    // (selection scratch and counters, under 3 KB)
+    return DecodePlanIn{d.dtype, d.d_model, d.n_experts, TS, di.sms, d.act == PP_ACT_SWIGLU, di.smem_optin - 4096};
+}
+
+// Largest token count one fused decode launch takes for this shape (0: none).
+int decode_ts_limit(const pp_desc& d) {
+    for (int ts = decode_max_ts(d.dtype); ts >= 1; ts >>= 1) {
+        DecodePlan plan;
+        if (decode_plan(plan_in(d, ts), &plan)) return ts;
+    }
+    return 0;
+}
+
 // One launch of the fused decode kernel over tokens [t0, t0 + n).
 pp_status decode_call(const pp_desc& d, const void* x, int t0, int n, const void* Wr, const void* Wg,
                       const void* Wu, const void* Wd, float p, const pp_selection* sel, bool do_route,
@@ -180,10 +196,8 @@ pp_status decode_call(const pp_desc& d, const void* x, int t0, int n, const void
     int TS = 1;
     while (TS < n) TS <<= 1;
     if (TS > decode_max_ts(d.dtype)) return PP_ERR_SHAPE;
-    // leave 2 KB of the opt-in limit for the kernel's static shared memory
-    DecodePlanIn in{d.dtype, d.d_model, d.n_experts, TS, di.sms, d.act == PP_ACT_SWIGLU, di.smem_optin - 2048};
     DecodePlan plan;
-    if (!decode_plan(in, &plan)) return PP_ERR_SHAPE;
+    if (!decode_plan(plan_in(d, TS), &plan)) return PP_ERR_SHAPE;
     DecodeArgs a;
     std::memset(&a, 0, sizeof a);
     const size_t esz = d.dtype == PP_BF16 ? 2 : 4;
@@ -214,16 +228,17 @@ pp_status decode_call(const pp_desc& d, const void* x, int t0, int n, const void
     a.p = p;
     a.do_route = do_route ? 1 : 0;
     a.do_ffn = do_ffn ? 1 : 0;
-    a.sel_slots = sel_slots_for(d.n_experts);
     a.R6 = plan.R6;
     a.NS4 = plan.NS4;
+    a.ded6 = plan.ded6;
+    a.slots6 = plan.slots6;
     a.uch = plan.uch;
     a.off_x = plan.off_x;
     a.off_gw = plan.off_gw;
     a.off_mask = plan.off_mask;
     a.off_ulist = plan.off_ulist;
     a.off_red = plan.off_red;
-    a.off_h = plan.off_h;
+    a.off_red6 = plan.off_red6;
     a.off_ring6 = plan.off_ring6;
     a.off_ring4 = plan.off_ring4;
     return cuda_status(decode_launch(a, plan, d.dtype, TS, di.sms, st));
@@ -276,7 +291,9 @@ pp_status pp_route(const pp_desc* desc, const void* x, int T, const void* W_r, f
     if (T == 0) return PP_OK;
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     const Ws w = ws_views(*desc, T, ws);
-    if (T <= decode_max_ts(desc->dtype))
+    const int ts = decode_ts_limit(*desc);
+    if (ts == 0) return PP_ERR_SHAPE;
+    if (T <= ts)
         return decode_call(*desc, x, 0, T, W_r, nullptr, nullptr, nullptr, p, out, true, false, nullptr, w, st);
     float* lg = out->logits ? out->logits : w.logits;
     PP_TRY(cuda_status(router_launch(desc->dtype, x, T, desc->d_model, W_r, desc->n_experts, lg, st)));
@@ -298,7 +315,8 @@ pp_status pp_sparse_ffn(const pp_desc* desc, const void* x, int T, const void* W
     if (T == 0) return PP_OK;
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     const Ws w = ws_views(*desc, T, ws);
-    const int ts = decode_max_ts(desc->dtype);
+    const int ts = decode_ts_limit(*desc);
+    if (ts == 0) return PP_ERR_SHAPE;
     for (int t0 = 0; t0 < T; t0 += ts) {
         const int n = std::min(ts, T - t0);
         PP_TRY(decode_call(*desc, x, t0, n, nullptr, W_gate, W_up, W_down, 0.0f, sel, false, true, y, w, st));
@@ -321,14 +339,15 @@ pp_status pp_layer(const pp_desc* desc, const void* x, int T, const void* W_r, c
     if (T == 0) return PP_OK;
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     const Ws w = ws_views(*desc, T, ws);
-    if (T <= decode_max_ts(desc->dtype))
+    const int ts = decode_ts_limit(*desc);
+    if (ts == 0) return PP_ERR_SHAPE;
+    if (T <= ts)
         return decode_call(*desc, x, 0, T, W_r, W_gate, W_up, W_down, p, sel_out, true, true, y, w, st);
     pp_selection s = sel_out ? *sel_out : pp_selection{w.ids, w.counts, w.gates, nullptr};
     float* lg = s.logits ? s.logits : w.logits;
     PP_TRY(cuda_status(router_launch(desc->dtype, x, T, desc->d_model, W_r, desc->n_experts, lg, st)));
     PP_TRY(cuda_status(select_launch(lg, T, desc->n_experts, p, desc->rule, desc->gate, s.ids, s.counts, s.gates,
                                      &w.ctrl->status, st)));
-    const int ts = decode_max_ts(desc->dtype);
     for (int t0 = 0; t0 < T; t0 += ts) {
         const int n = std::min(ts, T - t0);
         PP_TRY(decode_call(*desc, x, t0, n, nullptr, W_gate, W_up, W_down, 0.0f, &s, false, true, y, w, st));

@@ -1,76 +1,42 @@
 // Fused decode layer for small token counts (PrunePath Sec. 3.1 end to end).
 //
-// One cooperative, persistent launch of one CTA per SM does, for T <= TS
-// tokens:
+// One cooperative, persistent launch of one CTA (8 warps) per SM does, for
+// T <= TS tokens:
 //   phase 1  router (Eq. routing_logits): CTA b bulk-loads its rows of W_r
 //            and dots them with x (fp32 FMA), writing logits to the workspace;
 //   -- grid barrier --
-//   select   every CTA redundantly runs the warp selection of each token
-//            (Eq. softmax_prob, the descending order, Eq. tau_thresh_activate)
-//            and forms U, the union of the tokens' activated experts;
-//   phase 4  gate/up (Eq. ffn on the expert blocks): the U*64 neurons are
-//            split evenly over the grid; each consumer warp bulk-loads the
-//            gate and up rows of one neuron into its own shared-memory slot,
-//            computes h = act(.) * gate weight (Eq. moe_output) per token and
-//            stores it to the workspace;
+//   select   every CTA redundantly selects each token's experts with the
+//            CTA-parallel counting selection (Eq. softmax_prob, the
+//            descending order, Eq. tau_thresh_activate) and forms U, the
+//            union of the tokens' activated experts;
+//   phase 4  gate/up (Eq. ffn on the expert blocks): the |U|*64 neurons are
+//            split evenly over the grid; each warp bulk-loads the gate and up
+//            rows of one neuron into its own shared-memory slot, computes
+//            h = act(.) * gate weight (Eq. moe_output) per token and stores
+//            it to the workspace;
 //   -- grid barrier --
-//   phase 6  down projection: CTA b owns R6 rows of W_down and y; a producer
-//            warp streams the [R6 x 64] column block of every expert in U
-//            with 2-D tensor TMA (these loads are issued before phase 4 runs,
-//            so they overlap it), the consumer warps accumulate
-//            y[t][row] = sum_u sum_n W_down[row][u*64+n] * h[u][t][n] in fp32
-//            in registers and write y once (no atomics, deterministic).
+//   phase 6  down projection: CTA b owns R6 rows of W_down and y.  Warp w
+//            handles the experts u = w, w+8, ... of U: it streams the
+//            [R6 x 64] column block of each with 2-D tensor TMA into its own
+//            slots (the first ones are issued before phase 4, so they
+//            overlap it) and accumulates every row of the CTA in registers;
+//            one cross-warp reduction in shared memory then writes y once
+//            (no atomics: deterministic).
 // Only the selected expert blocks are read from HBM.
 #include "pp_common.cuh"
-#include "pp_select.cuh"
 #include "pp_kernels.h"
+#include "pp_select.cuh"
 
 namespace pp {
 
-constexpr int kConsumerWarps = 8;
-constexpr int kDecThreads = (kConsumerWarps + 1) * 32;
-constexpr int kNS6 = 8;   // phase-6 ring slots
-constexpr int kMaxNS4 = kConsumerWarps;
+constexpr int kWarps = 8;
+constexpr int kDecThreads = kWarps * 32;
+constexpr int kMaxNS4 = kWarps;
+constexpr int kMaxSlots6 = 4;  // phase-6 slots per warp
 
 // barrier indices in the first bytes of shared memory
-constexpr int kBarX = 0, kBarR = 1, kBarFull4 = 2, kBarFull6 = kBarFull4 + kMaxNS4,
-              kBarEmpty6 = kBarFull6 + kNS6, kNumBars = kBarEmpty6 + kNS6;
-
-template <typename TW, int TS, int S>
-PP_DEVINL void select_tokens(const DecodeArgs& a, float* gw, unsigned* mask, bool cta0) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int E = a.E;
-    if (warp >= a.T) return;
-    const int t = warp;
-    unsigned long long key[S];
-    bool finite = true;
-    const float* row = a.logit_ws + (size_t)t * E;
-    const int k = warp_select<S>([&](int j) { return __ldcg(row + j); }, E, a.p, a.rule, key, &finite);
-    if (!finite) {
-        if (lane == 0) record_status(a.status, PP_ERR_NONFINITE);
-    }
-#pragma unroll
-    for (int s = 0; s < S; s++) {
-        const int r = lane * S + s;
-        if (r >= E) continue;
-        const bool on = finite && r < k;
-        const int e = finite ? key_index(key[s]) : r;
-        const float gv = on ? gate_of(a.gate, key[s]) : 0.0f;
-        if (on) {
-            gw[t * E + e] = gv;
-            atomicOr(&mask[e], 1u << t);
-        }
-        if (cta0 && a.sel_ids) {
-            a.sel_ids[(size_t)t * E + r] = on ? e : -1;
-            a.sel_gates[(size_t)t * E + r] = gv;
-        }
-    }
-    if (cta0) {
-        if (a.sel_counts && lane == 0) a.sel_counts[t] = k;
-        if (a.sel_logits)
-            for (int j = lane; j < E; j += 32) a.sel_logits[(size_t)t * E + j] = __ldcg(row + j);
-    }
-}
+constexpr int kBarX = 0, kBarR = 1, kBarH = 2, kBarFull4 = 3, kBarFull6 = kBarFull4 + kMaxNS4,
+              kNumBars = kBarFull6 + kWarps * kMaxSlots6;
 
 // Selection given by the caller (pp_sparse_ffn): gates are summed per expert
 // so repeated ids behave like repeated terms of the sum.
@@ -94,13 +60,12 @@ PP_DEVINL void load_given_selection(const DecodeArgs& a, float* gw, unsigned* ma
     }
 }
 
-template <typename TW, int TS>
+template <typename TW, int TS, int RPL>
 __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __grid_constant__ DecodeArgs a) {
     extern __shared__ __align__(1024) unsigned char smem[];
     using EL = Elem<TW>;
     constexpr int kEl = EL::kPer16B;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const bool is_producer = warp == kConsumerWarps;
     const int T = a.T, d = a.d, E = a.E;
     const int G = gridDim.x, b = blockIdx.x;
     const int nchunk = d / kEl;  // 16-byte chunks per row
@@ -114,19 +79,19 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     unsigned* mask = reinterpret_cast<unsigned*>(smem + a.off_mask);
     int* ulist = reinterpret_cast<int*>(smem + a.off_ulist);
     float* red = reinterpret_cast<float*>(smem + a.off_red);
-    float* hs = reinterpret_cast<float*>(smem + a.off_h);
+    float* red6 = reinterpret_cast<float*>(smem + a.off_red6);
     unsigned char* ring4 = smem + a.off_ring4;
     unsigned char* ring6 = smem + a.off_ring6;
+    __shared__ __align__(16) CtaSelScratch sel_sc;
     __shared__ int s_nU;
-    __shared__ int s_wcount[kConsumerWarps + 1];
+    __shared__ int s_wcount[kWarps];
 
     if (tid == 0) {
-        for (int i = 0; i < kNumBars; i++)
-            mbar_init(&bars[i], (i >= kBarEmpty6) ? kConsumerWarps : 1);
+        for (int i = 0; i < kNumBars; i++) mbar_init(&bars[i], 1);
         fence_mbar_init();
     }
-    for (int i = tid; i < TS * E; i += blockDim.x) gw[i] = 0.0f;
-    for (int i = tid; i < kMaxExperts; i += blockDim.x) mask[i] = 0u;
+    for (int i = tid; i < TS * E; i += kDecThreads) gw[i] = 0.0f;
+    for (int i = tid; i < kMaxExperts; i += kDecThreads) mask[i] = 0u;
     __syncthreads();
 
     // this CTA's router rows [j0, j1) of W_r (phase 1)
@@ -135,7 +100,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     const int nrows = a.do_route ? max(0, j1 - j0) : 0;
 
     // x -> shared memory (all T rows are contiguous), and the router rows
-    if (is_producer && lane == 0) {
+    if (tid == 0) {
         const uint32_t bytes = (uint32_t)(T * rowb);
         mbar_arrive_expect_tx(&bars[kBarX], bytes);
         bulk_g2s(xs, a.x, bytes, &bars[kBarX]);
@@ -152,7 +117,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
 
     // ---------------------------------------------------------- phase 1
     if (a.do_route) {
-        if (!is_producer && nrows > 0) {
+        if (nrows > 0) {
             mbar_wait(&bars[kBarR], 0, a.status, lim);
             const TW* rows_s = reinterpret_cast<const TW*>(ring4);
             for (int r0 = 0; r0 < nrows; r0 += 2) {
@@ -161,7 +126,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
                 for (int i = 0; i < 2; i++)
 #pragma unroll
                     for (int t = 0; t < TS; t++) acc[i][t] = 0.0f;
-                for (int c = tid; c < nchunk; c += kConsumerWarps * 32) {
+                for (int c = tid; c < nchunk; c += kDecThreads) {
                     float xf[TS][kEl];
 #pragma unroll
                     for (int t = 0; t < TS; t++)
@@ -185,23 +150,44 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
                         const float v = warp_sum(acc[i][t]);
                         if (lane == 0) red[(warp * 2 + i) * TS + t] = v;
                     }
-                named_bar_sync(1, kConsumerWarps * 32);
+                __syncthreads();
                 if (tid < 2 * TS) {
                     const int i = tid / TS, t = tid % TS;
                     if (r0 + i < nrows && t < T) {
                         float v = 0.0f;
-                        for (int w = 0; w < kConsumerWarps; w++) v += red[(w * 2 + i) * TS + t];
+                        for (int w = 0; w < kWarps; w++) v += red[(w * 2 + i) * TS + t];
                         a.logit_ws[(size_t)t * E + j0 + r0 + i] = v;
                     }
                 }
-                named_bar_sync(1, kConsumerWarps * 32);
+                __syncthreads();
             }
         }
         grid_barrier(a.bar, a.status, lim);
-        if (a.sel_slots == 1) select_tokens<TW, TS, 1>(a, gw, mask, b == 0);
-        else if (a.sel_slots == 2) select_tokens<TW, TS, 2>(a, gw, mask, b == 0);
-        else if (a.sel_slots == 4) select_tokens<TW, TS, 4>(a, gw, mask, b == 0);
-        else select_tokens<TW, TS, 8>(a, gw, mask, b == 0);
+        // selection of every token by the whole CTA; CTA 0 publishes it
+        const bool publish = b == 0;
+        for (int t = 0; t < T; t++) {
+            bool on;
+            int r;
+            float g;
+            const int k = cta_select(a.logit_ws + (size_t)t * E, E, a.p, a.rule, sel_sc, a.status, &on, &r, &g);
+            const int j = tid;
+            if (j < E) {
+                const float gv = on ? (a.gate == PP_GATE_NONE ? 1.0f : sigmoidf_(g)) : 0.0f;
+                if (on) {
+                    gw[t * E + j] = gv;
+                    mask[j] |= 1u << t;
+                }
+                if (publish) {
+                    if (a.sel_ids) {
+                        a.sel_ids[(size_t)t * E + r] = on ? j : -1;
+                        a.sel_gates[(size_t)t * E + r] = gv;
+                    }
+                    if (a.sel_logits) a.sel_logits[(size_t)t * E + j] = g;
+                }
+            }
+            if (publish && tid == 0 && a.sel_counts) a.sel_counts[t] = k;
+            __syncthreads();  // scratch reuse by the next token
+        }
     } else {
         load_given_selection(a, gw, mask);
     }
@@ -217,7 +203,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
         __syncthreads();
         if (tid == 0) {
             int acc = 0;
-            for (int w = 0; w <= kConsumerWarps; w++) {
+            for (int w = 0; w < kWarps; w++) {
                 const int c = s_wcount[w];
                 s_wcount[w] = acc;
                 acc += c;
@@ -230,56 +216,61 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     }
     const int nU = s_nU;
 
-    // phase-6 geometry: CTA b owns rows [r0, r0 + rows) of W_down and y
+    // phase-6 geometry: CTA b owns rows [r0, r0 + rows) of W_down and y;
+    // warp w handles experts u = w + 8 i of U (i < nt_w)
     const int R6 = a.R6;
     const int r0 = b * R6;
     const int rows = max(0, min(R6, d - r0));
     const uint32_t stage6 = (uint32_t)(R6 * kDExpert * sizeof(TW));
     const int ntiles = rows > 0 ? nU : 0;
-
-    // producer: prefetch the first phase-6 tiles now, so they stream while
-    // phase 4 runs
-    if (is_producer && lane == 0) {
-        fence_proxy_async_smem();
-        for (int u = 0; u < min(ntiles, kNS6); u++) {
-            mbar_arrive_expect_tx(&bars[kBarFull6 + u], stage6);
-            tma_load_2d(ring6 + (size_t)u * stage6, &a.tmap_down, ulist[u] * kDExpert, r0,
-                        &bars[kBarFull6 + u]);
-        }
-    }
+    const int nt_w = ntiles > warp ? (ntiles - warp + kWarps - 1) / kWarps : 0;
+    const int ded6 = a.ded6, slots6 = a.slots6;
+    // a warp's first ded6 slots are its own part of the phase-6 ring; the
+    // others are carved from the phase-4 ring, free after the second barrier
+    auto slot6 = [&](int s) -> unsigned char* {
+        return s < ded6 ? ring6 + (size_t)(warp * ded6 + s) * stage6
+                        : ring4 + (size_t)(warp * (slots6 - ded6) + (s - ded6)) * stage6;
+    };
+    auto issue6 = [&](int i) {
+        const int s = i % slots6;
+        uint64_t* fb = &bars[kBarFull6 + warp * kMaxSlots6 + s];
+        mbar_arrive_expect_tx(fb, stage6);
+        tma_load_2d(slot6(s), &a.tmap_down, ulist[warp + kWarps * i] * kDExpert, r0, fb);
+    };
 
     // ---------------------------------------------------------- phase 4
     const int Ntot = nU * kDExpert;
     const int nb = (int)(((long long)b * Ntot) / G);
     const int ne = (int)(((long long)(b + 1) * Ntot) / G);
     const int cnt = ne - nb;
-    if (!is_producer && warp < a.NS4 && cnt > warp) {
-        const uint32_t stage4 = (uint32_t)((gated ? 2 : 1) * rowb);
-        unsigned char* slot = ring4 + (size_t)warp * stage4;
-        uint64_t* fb = &bars[kBarFull4 + warp];
-        const TW* Wg = reinterpret_cast<const TW*>(a.Wg);
-        const TW* Wu = reinterpret_cast<const TW*>(a.Wu);
-        auto issue = [&](int i) {
-            const int q = nb + i;
-            const int e = ulist[q >> 6];
-            const size_t row = (size_t)e * kDExpert + (q & 63);
-            mbar_arrive_expect_tx(fb, stage4);
-            if (gated) {
-                bulk_g2s(slot, Wg + row * d, (uint32_t)rowb, fb);
-                bulk_g2s(slot + rowb, Wu + row * d, (uint32_t)rowb, fb);
-            } else {
-                bulk_g2s(slot, Wu + row * d, (uint32_t)rowb, fb);
-            }
-        };
-        if (lane == 0) {
-            fence_proxy_async_smem();
-            issue(warp);
+    const bool ph4 = warp < a.NS4 && cnt > warp;
+    const uint32_t stage4 = (uint32_t)((gated ? 2 : 1) * rowb);
+    unsigned char* slot4 = ring4 + (size_t)warp * stage4;
+    uint64_t* fb4 = &bars[kBarFull4 + warp];
+    const TW* Wg = reinterpret_cast<const TW*>(a.Wg);
+    const TW* Wu = reinterpret_cast<const TW*>(a.Wu);
+    auto issue4 = [&](int i) {
+        const int q = nb + i;
+        const size_t row = (size_t)ulist[q >> 6] * kDExpert + (q & 63);
+        mbar_arrive_expect_tx(fb4, stage4);
+        if (gated) {
+            bulk_g2s(slot4, Wg + row * d, (uint32_t)rowb, fb4);
+            bulk_g2s(slot4 + rowb, Wu + row * d, (uint32_t)rowb, fb4);
+        } else {
+            bulk_g2s(slot4, Wu + row * d, (uint32_t)rowb, fb4);
         }
+    };
+    if (lane == 0) {
+        fence_proxy_async_smem();
+        if (ph4) issue4(warp);
+        for (int i = 0; i < min(nt_w, ded6); i++) issue6(i);  // phase-6 prefetch
+    }
+    if (ph4) {
         uint32_t use = 0;
-        const TW* gs = reinterpret_cast<const TW*>(slot);
-        const TW* us = reinterpret_cast<const TW*>(gated ? slot + rowb : slot);
+        const TW* gs = reinterpret_cast<const TW*>(slot4);
+        const TW* us = reinterpret_cast<const TW*>(gated ? slot4 + rowb : slot4);
         for (int i = warp; i < cnt; i += a.NS4) {
-            mbar_wait(fb, use & 1u, a.status, lim);
+            mbar_wait(fb4, use & 1u, a.status, lim);
             use++;
             float au[TS], ag[TS];
 #pragma unroll
@@ -316,7 +307,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
             __syncwarp();
             if (lane == 0 && i + a.NS4 < cnt) {
                 fence_proxy_async_smem();
-                issue(i + a.NS4);
+                issue4(i + a.NS4);
             }
         }
     }
@@ -324,81 +315,111 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     grid_barrier(a.bar, a.status, lim);
 
     // ---------------------------------------------------------- phase 6
-    if (is_producer) {
-        if (lane == 0) {
-            for (int u = kNS6; u < ntiles; u++) {
-                const int s = u % kNS6;
-                const uint32_t k = (uint32_t)(u / kNS6);
-                mbar_wait(&bars[kBarEmpty6 + s], (k - 1u) & 1u, a.status, lim);
-                fence_proxy_async_smem();
-                mbar_arrive_expect_tx(&bars[kBarFull6 + s], stage6);
-                tma_load_2d(ring6 + (size_t)s * stage6, &a.tmap_down, ulist[u] * kDExpert, r0,
-                            &bars[kBarFull6 + s]);
-            }
-        }
-        return;
-    }
     if (rows == 0) return;
+    // h of the first chunk of U -> shared memory (after the extra tile slots)
+    float* hs = reinterpret_cast<float*>(ring4 + (size_t)kWarps * (slots6 - ded6) * stage6);
+    const int uch = a.uch;  // experts per h chunk, a multiple of 8
+    const uint32_t hbytes_per_u = (uint32_t)(T * kDExpert * 4);
+    if (tid == 0 && ntiles > 0) {
+        fence_proxy_async_smem();
+        const uint32_t nbytes = (uint32_t)min(uch, ntiles) * hbytes_per_u;
+        mbar_arrive_expect_tx(&bars[kBarH], nbytes);
+        bulk_g2s(hs, a.h_ws, nbytes, &bars[kBarH]);
+    }
+    if (lane == 0) {
+        fence_proxy_async_smem();
+        for (int i = ded6; i < min(nt_w, slots6); i++) issue6(i);
+    }
+    if (ntiles > 0) mbar_wait(&bars[kBarH], 0, a.status, lim);
 
-    // consumer warp w accumulates row groups w and w + 8 (4 rows per group,
-    // 8 lanes per row, each lane a 16-byte chunk of the 64-wide block)
-    constexpr int kChunksPerRow = kDExpert / kEl;       // 8 (bf16) or 16 (fp32)
-    constexpr int kChunksPerLane = kChunksPerRow / 8;   // 1 or 2
-    const int sub = lane & 7;
-    const int rig = lane >> 3;
-    float acc[2][TS];
+    // lane: chunk column c of the 64-wide block (8 elements; fp32 uses two
+    // 4-element chunks c and c + 8) and rows rig + 4 j
+    constexpr int kCPL = kDExpert / kEl / 8;  // 16-byte chunks per lane per row: 1 (bf16) or 2 (fp32)
+    const int c = lane & 7, rig = lane >> 3;
+    float acc[RPL][TS];
 #pragma unroll
-    for (int i = 0; i < 2; i++)
+    for (int j = 0; j < RPL; j++)
 #pragma unroll
-        for (int t = 0; t < TS; t++) acc[i][t] = 0.0f;
-    const int uch = a.uch;
-    for (int u = 0; u < ntiles; u++) {
-        if (u % uch == 0) {
-            named_bar_sync(1, kConsumerWarps * 32);
-            const int nu = min(uch, ntiles - u);
-            const float4* src = reinterpret_cast<const float4*>(a.h_ws + (size_t)u * T * kDExpert);
-            float4* dst = reinterpret_cast<float4*>(hs);
-            for (int i = tid; i < nu * T * kDExpert / 4; i += kConsumerWarps * 32) dst[i] = __ldcg(src + i);
-            named_bar_sync(1, kConsumerWarps * 32);
+        for (int t = 0; t < TS; t++) acc[j][t] = 0.0f;
+    const int nt_all = (ntiles + kWarps - 1) / kWarps;  // same trip count in every warp
+    int hchunk = 0;
+    for (int i = 0; i < nt_all; i++) {
+        const int u = warp + kWarps * i;
+        if (kWarps * i >= (hchunk + 1) * uch) {  // next h chunk (uniform over the CTA)
+            __syncthreads();
+            hchunk++;
+            if (tid == 0) {
+                fence_proxy_async_smem();
+                const uint32_t nbytes = (uint32_t)min(uch, ntiles - hchunk * uch) * hbytes_per_u;
+                mbar_arrive_expect_tx(&bars[kBarH], nbytes);
+                bulk_g2s(hs, a.h_ws + (size_t)hchunk * uch * T * kDExpert, nbytes, &bars[kBarH]);
+            }
+            mbar_wait(&bars[kBarH], (uint32_t)hchunk & 1u, a.status, lim);
         }
-        const int s = u % kNS6;
-        mbar_wait(&bars[kBarFull6 + s], (uint32_t)(u / kNS6) & 1u, a.status, lim);
-        const TW* tile = reinterpret_cast<const TW*>(ring6 + (size_t)s * stage6);
-        const float* hu = hs + (size_t)(u % uch) * T * kDExpert;
+        if (i >= nt_w) continue;
+        const int s = i % slots6;
+        mbar_wait(&bars[kBarFull6 + warp * kMaxSlots6 + s], (uint32_t)(i / slots6) & 1u, a.status, lim);
+        const TW* tile = reinterpret_cast<const TW*>(slot6(s));
+        const float* hu = hs + (size_t)(u - hchunk * uch) * T * kDExpert;
+        float hv[TS][kCPL * kEl];
 #pragma unroll
-        for (int gi = 0; gi < 2; gi++) {
-            const int row = (warp + gi * kConsumerWarps) * 4 + rig;
+        for (int t = 0; t < TS; t++)
+            if (t < T)
+#pragma unroll
+                for (int cc = 0; cc < kCPL; cc++) {
+                    const float4* h4 =
+                        reinterpret_cast<const float4*>(hu + (size_t)t * kDExpert + (c + 8 * cc) * kEl);
+#pragma unroll
+                    for (int q4 = 0; q4 < kEl / 4; q4++) {
+                        const float4 v = h4[q4];
+                        hv[t][cc * kEl + q4 * 4 + 0] = v.x;
+                        hv[t][cc * kEl + q4 * 4 + 1] = v.y;
+                        hv[t][cc * kEl + q4 * 4 + 2] = v.z;
+                        hv[t][cc * kEl + q4 * 4 + 3] = v.w;
+                    }
+                }
+#pragma unroll
+        for (int j = 0; j < RPL; j++) {
+            const int row = rig + 4 * j;
             if (row < rows) {
 #pragma unroll
-                for (int cc = 0; cc < kChunksPerLane; cc++) {
-                    const int chunk = sub + cc * 8;
+                for (int cc = 0; cc < kCPL; cc++) {
                     float wf[kEl];
-                    EL::unpack(reinterpret_cast<const uint4*>(tile + (size_t)row * kDExpert)[chunk], wf);
+                    EL::unpack(reinterpret_cast<const uint4*>(tile + (size_t)row * kDExpert)[c + 8 * cc], wf);
 #pragma unroll
-                    for (int t = 0; t < TS; t++) {
-                        if (t < T) {
-                            const float* hv = hu + (size_t)t * kDExpert + chunk * kEl;
+                    for (int t = 0; t < TS; t++)
+                        if (t < T)
 #pragma unroll
-                            for (int q = 0; q < kEl; q++) acc[gi][t] = fmaf(wf[q], hv[q], acc[gi][t]);
-                        }
-                    }
+                            for (int q = 0; q < kEl; q++) acc[j][t] = fmaf(wf[q], hv[t][cc * kEl + q], acc[j][t]);
                 }
             }
         }
         __syncwarp();
-        if (lane == 0) mbar_arrive(&bars[kBarEmpty6 + s]);
+        if (lane == 0 && i + slots6 < nt_w) {
+            fence_proxy_async_smem();
+            issue6(i + slots6);
+        }
     }
+    // reduce over the 8 lanes of a row, then over the warps (fixed order)
 #pragma unroll
-    for (int gi = 0; gi < 2; gi++) {
-        const int row = (warp + gi * kConsumerWarps) * 4 + rig;
+    for (int j = 0; j < RPL; j++) {
+        const int row = rig + 4 * j;
 #pragma unroll
         for (int t = 0; t < TS; t++) {
-            float v = acc[gi][t];
+            float v = acc[j][t];
             v += __shfl_xor_sync(kFull, v, 1);
             v += __shfl_xor_sync(kFull, v, 2);
             v += __shfl_xor_sync(kFull, v, 4);
-            if (sub == 0 && row < rows && t < T) EL::store(a.y, (size_t)t * d + r0 + row, v);
+            if (c == 0 && row < rows && t < T) red6[(warp * R6 + row) * TS + t] = v;
         }
+    }
+    __syncthreads();
+    for (int o = tid; o < rows * T; o += kDecThreads) {
+        const int row = o / T, t = o % T;
+        float v = 0.0f;
+        for (int w = 0; w < kWarps; w++)
+            if (w < ntiles) v += red6[(w * R6 + row) * TS + t];
+        EL::store(a.y, (size_t)t * d + r0 + row, v);
     }
 }
 
@@ -415,7 +436,11 @@ bool decode_plan(const DecodePlanIn& in, DecodePlan* out) {
     const int G = in.grid;
     DecodePlan p{};
     p.R6 = (in.d + G - 1) / G;
-    if (p.R6 > 2 * kConsumerWarps * 4) return false;  // 64 rows per CTA at most
+    if (p.R6 > 64) return false;  // 64 rows per CTA at most (16 per lane)
+    p.RPL = (p.R6 + 3) / 4 <= 8 ? 8 : 16;
+    const size_t stage6 = (size_t)p.R6 * kDExpert * esz;
+    const size_t stage4 = (size_t)(in.gated ? 2 : 1) * in.d * esz;
+    const int rpc = (in.E + G - 1) / G;
     size_t off = align_up(kNumBars * 8, 128);
     p.off_x = (uint32_t)off;
     off = align_up(off + (size_t)TS * in.d * esz, 128);
@@ -426,32 +451,42 @@ bool decode_plan(const DecodePlanIn& in, DecodePlan* out) {
     p.off_ulist = (uint32_t)off;
     off = align_up(off + kMaxExperts * 4, 128);
     p.off_red = (uint32_t)off;
-    off = align_up(off + (size_t)kConsumerWarps * 2 * TS * 4, 128);
-    p.uch = (int)std::max<size_t>(1, (16 * 1024) / ((size_t)TS * kDExpert * 4));
-    if (p.uch > in.E) p.uch = in.E;
-    p.off_h = (uint32_t)off;
-    off = align_up(off + (size_t)p.uch * TS * kDExpert * 4, 1024);
-    p.off_ring6 = (uint32_t)off;
-    off = align_up(off + (size_t)kNS6 * p.R6 * kDExpert * esz, 1024);
-    p.off_ring4 = (uint32_t)off;
-    const size_t stage4 = (size_t)(in.gated ? 2 : 1) * in.d * esz;
+    off = align_up(off + (size_t)kWarps * 2 * TS * 4, 128);
+    p.off_red6 = (uint32_t)off;
+    off = align_up(off + (size_t)kWarps * p.R6 * TS * 4, 1024);
     const size_t budget = in.smem_limit;
+    // dedicated phase-6 slots: 2 per warp when they fit comfortably, else 1
+    p.ded6 = (off + 2 * kWarps * stage6 + 2 * stage4 <= budget) ? 2 : 1;
+    p.off_ring6 = (uint32_t)off;
+    off = align_up(off + (size_t)p.ded6 * kWarps * stage6, 1024);
+    p.off_ring4 = (uint32_t)off;
     if (off + stage4 > budget) return false;
-    int ns4 = (int)std::min<size_t>(kMaxNS4, (budget - off) / stage4);
-    // phase 1 reuses the ring for this CTA's router rows
-    const int rpc = (in.E + G - 1) / G;
-    while ((size_t)ns4 * stage4 < (size_t)rpc * in.d * esz && ns4 < kMaxNS4) ns4++;
-    if (off + (size_t)ns4 * stage4 > budget) return false;
+    const size_t avail = budget - off;
+    const int ns4 = (int)std::min<size_t>(kMaxNS4, avail / stage4);
+    // the ring also holds this CTA's router rows (phase 1) and, after phase
+    // 4, the extra phase-6 slots plus an h chunk of at least 8 experts
+    const size_t hper = (size_t)TS * kDExpert * 4;
+    size_t ring4 = 0;
+    int ext = kMaxSlots6 - p.ded6;
+    for (; ext >= 0; ext--) {
+        ring4 = std::max({(size_t)ns4 * stage4, (size_t)rpc * in.d * esz,
+                          (size_t)ext * kWarps * stage6 + 8 * hper});
+        if (ring4 <= avail) break;
+    }
+    if (ext < 0) return false;
+    p.slots6 = p.ded6 + ext;
+    const size_t harea = ring4 - (size_t)ext * kWarps * stage6;
+    p.uch = (int)(std::min<size_t>(kMaxExperts, harea / hper) / 8 * 8);
     p.NS4 = ns4;
-    p.smem = off + (size_t)ns4 * stage4;
+    p.smem = off + ring4;
     p.threads = kDecThreads;
     *out = p;
     return true;
 }
 
-template <typename TW, int TS>
+template <typename TW, int TS, int RPL>
 static cudaError_t launch_one(const DecodeArgs& a, const DecodePlan& p, int grid, cudaStream_t st) {
-    auto kern = decode_layer_kernel<TW, TS>;
+    auto kern = decode_layer_kernel<TW, TS, RPL>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg{};
@@ -467,21 +502,26 @@ static cudaError_t launch_one(const DecodeArgs& a, const DecodePlan& p, int grid
     return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
+template <typename TW, int TS>
+static cudaError_t launch_rpl(const DecodeArgs& a, const DecodePlan& p, int grid, cudaStream_t st) {
+    return p.RPL == 8 ? launch_one<TW, TS, 8>(a, p, grid, st) : launch_one<TW, TS, 16>(a, p, grid, st);
+}
+
 cudaError_t decode_launch(const DecodeArgs& a, const DecodePlan& p, int dtype, int TS, int grid,
                           cudaStream_t st) {
     if (dtype == PP_BF16) {
         switch (TS) {
-            case 1: return launch_one<__nv_bfloat16, 1>(a, p, grid, st);
-            case 2: return launch_one<__nv_bfloat16, 2>(a, p, grid, st);
-            case 4: return launch_one<__nv_bfloat16, 4>(a, p, grid, st);
+            case 1: return launch_rpl<__nv_bfloat16, 1>(a, p, grid, st);
+            case 2: return launch_rpl<__nv_bfloat16, 2>(a, p, grid, st);
+            case 4: return launch_rpl<__nv_bfloat16, 4>(a, p, grid, st);
             default: return cudaErrorInvalidValue;
         }
     }
     switch (TS) {
-        case 1: return launch_one<float, 1>(a, p, grid, st);
-        case 2: return launch_one<float, 2>(a, p, grid, st);
-        case 4: return launch_one<float, 4>(a, p, grid, st);
-        case 8: return launch_one<float, 8>(a, p, grid, st);
+        case 1: return launch_rpl<float, 1>(a, p, grid, st);
+        case 2: return launch_rpl<float, 2>(a, p, grid, st);
+        case 4: return launch_rpl<float, 4>(a, p, grid, st);
+        case 8: return launch_rpl<float, 8>(a, p, grid, st);
         default: return cudaErrorInvalidValue;
     }
 }

@@ -33,9 +33,8 @@ struct DecodeArgs {
     int act, gate, rule;
     float p;
     int do_route, do_ffn;
-    int sel_slots;         // keys per lane of the warp sort (E <= 32 * sel_slots)
-    int R6, NS4, uch;
-    uint32_t off_x, off_gw, off_mask, off_ulist, off_red, off_h, off_ring6, off_ring4;
+    int R6, NS4, ded6, slots6, uch;
+    uint32_t off_x, off_gw, off_mask, off_ulist, off_red, off_red6, off_ring6, off_ring4;
 };
 
 struct DecodePlanIn {
@@ -45,9 +44,9 @@ struct DecodePlanIn {
 };
 
 struct DecodePlan {
-    int R6, NS4, uch, threads;
+    int R6, RPL, NS4, ded6, slots6, uch, threads;
     size_t smem;
-    uint32_t off_x, off_gw, off_mask, off_ulist, off_red, off_h, off_ring6, off_ring4;
+    uint32_t off_x, off_gw, off_mask, off_ulist, off_red, off_red6, off_ring6, off_ring4;
 };
 
 bool decode_plan(const DecodePlanIn& in, DecodePlan* out);

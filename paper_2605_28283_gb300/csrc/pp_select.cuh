@@ -30,37 +30,53 @@ PP_DEVINL float key_logit(unsigned long long k) {
 
 PP_DEVINL int key_index(unsigned long long k) { return (int)(unsigned)(k & 0xffffffffull); }
 
+// One in-lane compare-exchange stage (partner slot s | STRIDE).
+template <int S, int STRIDE>
+PP_DEVINL void inlane_stage(unsigned long long (&key)[S], int lane, int size) {
+    if constexpr (STRIDE < S) {
+#pragma unroll
+        for (int s = 0; s < S; s++) {
+            if ((s & STRIDE) == 0) {
+                const int s2 = s | STRIDE;
+                const bool asc = ((lane * S + s) & size) == 0;
+                const unsigned long long a = key[s], b = key[s2];
+                const bool sw = asc ? (a > b) : (a < b);
+                key[s] = sw ? b : a;
+                key[s2] = sw ? a : b;
+            }
+        }
+    }
+}
+
+// Bitonic sort of the warp's 32*S keys into ascending order.  The stage
+// loops stay rolled (only the per-lane slot loop is unrolled): the network
+// is executed once per token, so compact code that stays in the
+// instruction cache beats straight-line code.
 template <int S>
 PP_DEVINL void warp_bitonic_sort(unsigned long long (&key)[S]) {
     const int lane = threadIdx.x & 31;
-#pragma unroll
+#pragma unroll 1
     for (int size = 2; size <= 32 * S; size <<= 1) {
-#pragma unroll
+#pragma unroll 1
         for (int stride = size >> 1; stride > 0; stride >>= 1) {
             if (stride >= S) {
                 const int ls = stride / S;
+                const bool lower = (lane & ls) == 0;
 #pragma unroll
                 for (int s = 0; s < S; s++) {
-                    const int i = lane * S + s;
+                    const bool asc = ((lane * S + s) & size) == 0;
                     const unsigned long long o = __shfl_xor_sync(kFull, key[s], ls);
-                    const bool take_min = ((i & stride) == 0) == ((i & size) == 0);
+                    const bool take_min = lower == asc;
                     const unsigned long long lo = key[s] < o ? key[s] : o;
                     const unsigned long long hi = key[s] < o ? o : key[s];
                     key[s] = take_min ? lo : hi;
                 }
+            } else if (stride == 4) {
+                inlane_stage<S, 4>(key, lane, size);
+            } else if (stride == 2) {
+                inlane_stage<S, 2>(key, lane, size);
             } else {
-#pragma unroll
-                for (int s = 0; s < S; s++) {
-                    if ((s & stride) == 0) {
-                        const int s2 = s | stride;
-                        const int i = lane * S + s;
-                        const bool asc = (i & size) == 0;
-                        const unsigned long long a = key[s], b = key[s2];
-                        const bool sw = asc ? (a > b) : (a < b);
-                        key[s] = sw ? b : a;
-                        key[s2] = sw ? a : b;
-                    }
-                }
+                inlane_stage<S, 1>(key, lane, size);
             }
         }
     }
@@ -126,6 +142,131 @@ PP_DEVINL int warp_select(Load load, int E, float p, int rule, unsigned long lon
 // Gate weight of the expert at a sorted key (Eq. moe_output).
 PP_DEVINL float gate_of(int gate_mode, unsigned long long k) {
     return gate_mode == PP_GATE_NONE ? 1.0f : sigmoidf_(key_logit(k));
+}
+
+// ---------------------------------------------------------------------------
+// CTA-parallel selection of one token (used where a single token's latency
+// matters).  Thread j owns expert j (E <= blockDim.x <= 256).  Instead of
+// sorting, every thread counts the experts ranked ahead of it (larger logit,
+// or equal logit and lower index) and sums their exponentials: its rank r_j
+// and the exclusive prefix mass S_{r_j - 1} in rank order.  The exponentials
+// e_j = exp(g_j - max g) (fp32) are summed as exact 2^-31 fixed-point
+// integers, and the cut compares S against p * Z exactly in integers, so
+// the only rounding is that of the fp32 exponentials.
+//   MIN_PREFIX: j selected  <=>  r_j == 0  or  S_{r_j - 1} <  p Z
+//   PAPER:      j selected  <=>  r_j == 0  or  S_{r_j}     <  p Z
+// (S non-decreasing along the order, so both are prefixes of the order.)
+
+struct CtaSelScratch {
+    uint32_t D[kMaxExperts];  // descending-order keys (ascending = larger logit)
+    uint32_t U[kMaxExperts];  // fixed-point exponentials, e * 2^31
+    float fred[8];
+    unsigned long long ured[8];
+};
+
+PP_DEVINL uint32_t desc_key(float g) {
+    unsigned u = __float_as_uint(g);
+    if ((u << 1) == 0u) u = 0u;
+    const unsigned ord = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+    return ~ord;
+}
+
+// Largest integer M with M * 2^sh < p_mant * Z, for p = p_mant * 2^-sh in
+// (0, 1); returns -1 (as a flag) when no prefix can be below p Z.
+PP_DEVINL long long prefix_threshold(float p, unsigned long long Z) {
+    if (!(p > 0.0f)) return -1;
+    const unsigned bits = __float_as_uint(p);
+    const unsigned ex = (bits >> 23) & 0xffu;
+    const unsigned long long mant = ex ? ((bits & 0x7fffffu) | 0x800000u) : (bits & 0x7fffffu);
+    const int sh = ex ? 150 - (int)ex : 149;
+    const unsigned long long rhs = mant * Z;  // < 2^24 * 2^39
+    if (rhs == 0ull) return -1;
+    if (sh >= 64) return 0;  // only an empty prefix (mass 0) is below p Z
+    return (long long)((rhs - 1ull) >> sh);
+}
+
+// Returns the activated count (CTA-uniform).  On return: *sel = whether
+// expert j (= threadIdx.x) is activated, *rank = its rank (valid j only),
+// *gval = its logit.  All threads of the CTA must call it.
+PP_DEVINL int cta_select(const float* __restrict__ logits_row, int E, float p, int rule,
+                         CtaSelScratch& sc, unsigned* status, bool* sel, int* rank,
+                         float* gval) {
+    const int j = threadIdx.x;
+    const int lane = j & 31, warp = j >> 5, nwarps = blockDim.x >> 5;
+    const bool valid = j < E;
+    const float g = valid ? __ldcg(logits_row + j) : -INFINITY;
+    *gval = g;
+    const bool fin = !valid || isfinite(g);
+    if (!__syncthreads_and(fin)) {
+        if (j == 0) record_status(status, PP_ERR_NONFINITE);
+        *sel = false;
+        *rank = j;
+        return 0;
+    }
+    // max logit
+    float m = g;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(kFull, m, o));
+    if (lane == 0) sc.fred[warp] = m;
+    __syncthreads();
+    m = sc.fred[0];
+    for (int w = 1; w < nwarps; w++) m = fmaxf(m, sc.fred[w]);
+    // fixed-point exponentials and their sum Z
+    const float e = valid ? expf(g - m) : 0.0f;
+    const uint32_t U = valid ? __float2uint_rn(e * 2147483648.0f) : 0u;
+    const uint32_t D = valid ? desc_key(g) : 0xffffffffu;
+    sc.D[j] = D;
+    sc.U[j] = U;
+    unsigned long long z = U;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(kFull, z, o);
+    if (lane == 0) sc.ured[warp] = z;
+    __syncthreads();
+    unsigned long long Z = 0;
+    for (int w = 0; w < nwarps; w++) Z += sc.ured[w];
+    // rank and exclusive prefix mass by counting the experts ahead: first the
+    // strictly larger logits, then (rare) equal logits with a lower index --
+    // equal logits have equal exponentials, so they add U once each
+    int r = 0, eq = 0;
+    unsigned long long ahead_mass = 0;
+    const int E4 = E & ~3;
+    for (int i = 0; i < E4; i += 4) {
+        const uint4 d4 = *reinterpret_cast<const uint4*>(&sc.D[i]);
+        const uint4 u4 = *reinterpret_cast<const uint4*>(&sc.U[i]);
+        const uint32_t dd[4] = {d4.x, d4.y, d4.z, d4.w};
+        const uint32_t uu[4] = {u4.x, u4.y, u4.z, u4.w};
+#pragma unroll
+        for (int q = 0; q < 4; q++) {
+            const bool lt = dd[q] < D;
+            r += lt ? 1 : 0;
+            eq += dd[q] == D ? 1 : 0;
+            ahead_mass += lt ? (unsigned long long)uu[q] : 0ull;
+        }
+    }
+    for (int i = E4; i < E; i++) {
+        const bool lt = sc.D[i] < D;
+        r += lt ? 1 : 0;
+        eq += sc.D[i] == D ? 1 : 0;
+        ahead_mass += lt ? (unsigned long long)sc.U[i] : 0ull;
+    }
+    if (valid && eq > 1) {  // ties: the equal logits of lower index are ahead
+        int tb = 0;
+        for (int i = 0; i < j; i++) tb += sc.D[i] == D ? 1 : 0;
+        r += tb;
+        ahead_mass += (unsigned long long)tb * U;
+    }
+    bool on;
+    if (p >= 1.0f) {
+        on = valid;
+    } else {
+        const long long thr = prefix_threshold(p, Z);
+        const unsigned long long mass = rule == PP_SEL_PAPER ? ahead_mass + U : ahead_mass;
+        on = valid && (r == 0 || (thr >= 0 && mass <= (unsigned long long)thr));
+    }
+    *sel = on;
+    *rank = r;
+    const int k = __syncthreads_count(on);
+    return k;
 }
 
 }  // namespace pp

@@ -32,10 +32,35 @@ __global__ void __launch_bounds__(256) select_kernel(const float* __restrict__ l
     if (lane == 0) counts[t] = k;
 }
 
+// One CTA per token (the latency-oriented counting selection of
+// pp_select.cuh); used for small token counts.
+__global__ void __launch_bounds__(256) select_cta_kernel(const float* __restrict__ logits, int E, float p,
+                                                         int rule, int gate, int32_t* ids, int32_t* counts,
+                                                         float* gates, unsigned* status) {
+    __shared__ __align__(16) CtaSelScratch sc;
+    const int t = blockIdx.x;
+    bool on;
+    int r;
+    float g;
+    const int k = cta_select(logits + (size_t)t * E, E, p, rule, sc, status, &on, &r, &g);
+    const int j = threadIdx.x;
+    if (j < E) {
+        ids[(size_t)t * E + r] = on ? j : -1;
+        gates[(size_t)t * E + r] = on ? (gate == PP_GATE_NONE ? 1.0f : sigmoidf_(g)) : 0.0f;
+    }
+    if (j == 0) counts[t] = k;
+}
+
+constexpr int kCtaSelectMaxT = 64;
+
 cudaError_t select_launch(const float* logits, int T, int E, float p, int rule, int gate,
                           int32_t* ids, int32_t* counts, float* gates, unsigned* status,
                           cudaStream_t st) {
     if (T == 0) return cudaSuccess;
+    if (T <= kCtaSelectMaxT) {
+        select_cta_kernel<<<T, 256, 0, st>>>(logits, E, p, rule, gate, ids, counts, gates, status);
+        return cudaGetLastError();
+    }
     const int warps = 8;
     const dim3 grid((T + warps - 1) / warps), block(32 * warps);
     switch (sel_slots_for(E)) {
