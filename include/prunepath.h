@@ -108,9 +108,9 @@ typedef struct pp_selection {
 /* Bytes of workspace needed for calls with up to T tokens. */
 size_t pp_workspace_size(const pp_desc *desc, int T);
 
-/* Zero the workspace's control words (status, barrier counters) on `stream`.
-   Call once after allocating a workspace, and again to clear a sticky
-   device error. */
+/* Zero the whole workspace (status word, barrier counters, accumulators) on
+   `stream`.  Call once after allocating a workspace, and again to clear a
+   sticky device error. */
 pp_status pp_workspace_init(void *ws, size_t ws_bytes, void *stream);
 
 /* Router and selection (Eq. routing_logits, softmax_prob,

@@ -43,41 +43,56 @@ DeviceInfo device_info() {
     return cache[dev];
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    static std::once_flag once;
-    std::call_once(once, [] {
-        void* p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-    });
-    return fn;
-}
-
 size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
+
+// Token counts above this use the tensor-core grouped path (bf16 only).
+constexpr int kGroupedMinT = 5;
+
+bool use_grouped(const pp_desc& d, int T) { return d.dtype == PP_BF16 && T >= kGroupedMinT; }
 
 // Workspace layout for calls with up to T tokens.
 struct Layout {
-    size_t logits, ids, counts, gates, h, total;
+    size_t logits, ids, counts, gates, h;
+    // grouped path
+    size_t part, bits, gexp, invpos, wcnt, blkcnt, blkbase, offsets, n_items, items, perm_token, perm_gate, H, Y,
+        yacc, overflow;
+    size_t total;
 };
 
 Layout layout(const pp_desc& d, int T) {
     const size_t E = (size_t)d.n_experts, Tn = (size_t)(T > 0 ? T : 1);
     Layout L{};
     size_t off = sizeof(Control);
-    L.logits = off;
-    off = align256(off + Tn * E * 4);
-    L.ids = off;
-    off = align256(off + Tn * E * 4);
-    L.counts = off;
-    off = align256(off + Tn * 4);
-    L.gates = off;
-    off = align256(off + Tn * E * 4);
-    L.h = off;
-    off = align256(off + E * 8 * kDExpert * 4);
+    auto take = [&](size_t bytes) {
+        const size_t at = off;
+        off = align256(off + bytes);
+        return at;
+    };
+    L.logits = take(Tn * E * 4);
+    L.ids = take(Tn * E * 4);
+    L.counts = take(Tn * 4);
+    L.gates = take(Tn * E * 4);
+    L.h = take(E * 8 * kDExpert * 4);
+    if (use_grouped(d, T)) {
+        const GroupedPlan g = grouped_plan(T, d.d_model, d.n_experts, 152);
+        L.part = take((size_t)g.nsplit * Tn * E * 4);
+        L.bits = take(Tn * 8 * 4);
+        L.gexp = take(Tn * E * 4);
+        L.invpos = take(Tn * E * 4);
+        const size_t nblk = (Tn + 255) / 256;
+        L.wcnt = take(nblk * 8 * E * 4);
+        L.blkcnt = take(nblk * E * 4);
+        L.blkbase = take(nblk * E * 4);
+        L.offsets = take((E + 1) * 4);
+        L.n_items = take(16);
+        L.items = take((size_t)g.max_items * 16);
+        L.perm_token = take((size_t)g.nnz_max * 4);
+        L.perm_gate = take((size_t)g.nnz_max * 4);
+        L.H = take(((size_t)g.nnz_max + 128) * kDExpert * 2);
+        L.Y = take((size_t)g.ycap * d.d_model * 2);
+        L.yacc = take(Tn * (size_t)d.d_model * 4);
+        L.overflow = take(16);
+    }
     L.total = off;
     return L;
 }
@@ -188,6 +203,50 @@ int decode_ts_limit(const pp_desc& d) {
     return 0;
 }
 
+GroupedArgs grouped_args(const pp_desc& d, int T, void* ws, const void* x, const void* Wr, const void* Wg,
+                         const void* Wu, const void* Wd, float p, const pp_selection& sel, void* y) {
+    const Layout L = layout(d, T);
+    char* b = static_cast<char*>(ws);
+    GroupedArgs a{};
+    a.plan = grouped_plan(T, d.d_model, d.n_experts, 152);
+    a.x = x;
+    a.Wr = Wr;
+    a.Wg = Wg;
+    a.Wu = Wu;
+    a.Wd = Wd;
+    a.y = y;
+    a.T = T;
+    a.d = d.d_model;
+    a.E = d.n_experts;
+    a.act = d.act;
+    a.gate = d.gate;
+    a.rule = d.rule;
+    a.p = p;
+    a.ids = sel.ids;
+    a.counts = sel.counts;
+    a.gates = sel.gates;
+    a.logits_out = sel.logits;
+    a.part = reinterpret_cast<float*>(b + L.part);
+    a.bits = reinterpret_cast<uint32_t*>(b + L.bits);
+    a.gexp = reinterpret_cast<float*>(b + L.gexp);
+    a.invpos = reinterpret_cast<int*>(b + L.invpos);
+    a.wcnt = reinterpret_cast<int*>(b + L.wcnt);
+    a.blkcnt = reinterpret_cast<int*>(b + L.blkcnt);
+    a.blkbase = reinterpret_cast<int*>(b + L.blkbase);
+    a.offsets = reinterpret_cast<int*>(b + L.offsets);
+    a.n_items = reinterpret_cast<int*>(b + L.n_items);
+    a.items = b + L.items;
+    a.perm_token = reinterpret_cast<int*>(b + L.perm_token);
+    a.perm_gate = reinterpret_cast<float*>(b + L.perm_gate);
+    a.H = reinterpret_cast<__nv_bfloat16*>(b + L.H);
+    a.Y = reinterpret_cast<__nv_bfloat16*>(b + L.Y);
+    a.yacc = reinterpret_cast<float*>(b + L.yacc);
+    a.overflow = reinterpret_cast<int*>(b + L.overflow);
+    a.status = &reinterpret_cast<Control*>(b)->status;
+    a.timeout_ns = kDefaultTimeoutNs;
+    return a;
+}
+
 // One launch of the fused decode kernel over tokens [t0, t0 + n).
 pp_status decode_call(const pp_desc& d, const void* x, int t0, int n, const void* Wr, const void* Wg,
                       const void* Wu, const void* Wd, float p, const pp_selection* sel, bool do_route,
@@ -245,6 +304,21 @@ pp_status decode_call(const pp_desc& d, const void* x, int t0, int n, const void
 }
 
 }  // namespace
+
+TensorMapEncodeFn tensor_map_encoder() {
+    static TensorMapEncodeFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<TensorMapEncodeFn>(p);
+    });
+    return fn;
+}
+
 }  // namespace pp
 
 using namespace pp;
@@ -258,7 +332,7 @@ size_t pp_workspace_size(const pp_desc* desc, int T) {
 
 pp_status pp_workspace_init(void* ws, size_t ws_bytes, void* stream) {
     if (!ws || ((uintptr_t)ws & 255u) != 0 || ws_bytes < sizeof(Control)) return PP_ERR_WORKSPACE;
-    return cuda_status(cudaMemsetAsync(ws, 0, sizeof(Control), static_cast<cudaStream_t>(stream)));
+    return cuda_status(cudaMemsetAsync(ws, 0, ws_bytes, static_cast<cudaStream_t>(stream)));
 }
 
 pp_status pp_select(const pp_desc* desc, const float* logits, int T, float p, const pp_selection* out,
@@ -291,6 +365,10 @@ pp_status pp_route(const pp_desc* desc, const void* x, int T, const void* W_r, f
     if (T == 0) return PP_OK;
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     const Ws w = ws_views(*desc, T, ws);
+    if (use_grouped(*desc, T)) {
+        const GroupedArgs a = grouped_args(*desc, T, ws, x, W_r, nullptr, nullptr, nullptr, p, *out, nullptr);
+        return cuda_status(grouped_route(a, st));
+    }
     const int ts = decode_ts_limit(*desc);
     if (ts == 0) return PP_ERR_SHAPE;
     if (T <= ts)
@@ -315,6 +393,10 @@ pp_status pp_sparse_ffn(const pp_desc* desc, const void* x, int T, const void* W
     if (T == 0) return PP_OK;
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     const Ws w = ws_views(*desc, T, ws);
+    if (use_grouped(*desc, T)) {
+        const GroupedArgs a = grouped_args(*desc, T, ws, x, nullptr, W_gate, W_up, W_down, 0.0f, *sel, y);
+        return cuda_status(grouped_ffn(a, device_info().sms, st));
+    }
     const int ts = decode_ts_limit(*desc);
     if (ts == 0) return PP_ERR_SHAPE;
     for (int t0 = 0; t0 < T; t0 += ts) {
@@ -339,11 +421,16 @@ pp_status pp_layer(const pp_desc* desc, const void* x, int T, const void* W_r, c
     if (T == 0) return PP_OK;
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     const Ws w = ws_views(*desc, T, ws);
+    pp_selection s = sel_out ? *sel_out : pp_selection{w.ids, w.counts, w.gates, nullptr};
+    if (use_grouped(*desc, T)) {
+        const GroupedArgs a = grouped_args(*desc, T, ws, x, W_r, W_gate, W_up, W_down, p, s, y);
+        PP_TRY(cuda_status(grouped_route(a, st)));
+        return cuda_status(grouped_ffn(a, device_info().sms, st));
+    }
     const int ts = decode_ts_limit(*desc);
     if (ts == 0) return PP_ERR_SHAPE;
     if (T <= ts)
         return decode_call(*desc, x, 0, T, W_r, W_gate, W_up, W_down, p, sel_out, true, true, y, w, st);
-    pp_selection s = sel_out ? *sel_out : pp_selection{w.ids, w.counts, w.gates, nullptr};
     float* lg = s.logits ? s.logits : w.logits;
     PP_TRY(cuda_status(router_launch(desc->dtype, x, T, desc->d_model, W_r, desc->n_experts, lg, st)));
     PP_TRY(cuda_status(select_launch(lg, T, desc->n_experts, p, desc->rule, desc->gate, s.ids, s.counts, s.gates,

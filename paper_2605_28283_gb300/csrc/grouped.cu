@@ -1,0 +1,752 @@
+// Tensor-core (tcgen05) path for many tokens: batched decode and prefill.
+//
+//   router GEMM   logits = X W_r^T (Eq. routing_logits), split over K; the
+//                 selection kernel sums the K-split partials in fixed order
+//   dispatch      per-token expert bitmasks -> per-expert counts -> offsets
+//                 and 128-row work items -> a stable permutation (tokens in
+//                 ascending order within each expert) with each assignment's
+//                 gate weight
+//   grouped G/U   per work item (expert e, <= 128 of its tokens):
+//                 D[128 x (64|128)] = X_gathered * [W_gate_e ; W_up_e]^T on
+//                 tcgen05 (TMA gather4 for the token rows), then
+//                 h = act(gate, up) * gate weight (Eq. ffn, Eq. moe_output),
+//                 stored bf16 in permuted order
+//   grouped down  per work item and 256-wide slice j of d:
+//                 D[128 x 256] = H_item * W_down[j, e-block]^T (K = 64); each
+//                 row (one token-expert assignment) is stored bf16 in the
+//                 permuted order
+//   combine       y[t] = sum over t's experts, in ascending expert order, of
+//                 its assignment rows (fp32 accumulation, deterministic)
+//   Assignments past the row buffer's capacity (only near-dense selections)
+//   are added into an fp32 accumulator with vector reductions instead; the
+//   combine step reads and re-zeroes it.
+//
+// Every GEMM kernel: warp 0 = TMA producer, warp 1 = TMEM owner and UMMA
+// issuer (one thread), warps 2..5 = epilogue (TMEM lanes 32*(warp%4)..).
+// All waits are bounded (PP_ERR_TIMEOUT).
+#include "pp_common.cuh"
+#include "pp_kernels.h"
+#include "pp_select.cuh"
+#include "pp_tc.cuh"
+
+namespace pp {
+
+constexpr int kTcThreads = 192;
+constexpr int kTileBytesA = 128 * 128;  // 128 rows x 64 bf16
+
+struct WorkItem {
+    int e, a0, cnt, pad;
+};
+
+// ====================================================================== router
+// Grid (m-tiles, splits).  CTA (m, s): D[128 tokens x NE] over K chunks
+// [s*kpb, min((s+1)*kpb, nk)); partial logits to part[s][t][e].
+template <int NE>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    router_gemm_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant__ CUtensorMap map_wr,
+                       int T, int E, int nk, int kpb, float* part, unsigned* status, uint64_t lim) {
+    constexpr int kStages = 4;
+    constexpr int kTileB = NE * 128;
+    constexpr int kStage = kTileBytesA + kTileB;
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    __shared__ uint64_t full[kStages], empty[kStages], tfull;
+    __shared__ uint32_t taddr_s;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.x * 128, split = blockIdx.y;
+    const int k0 = split * kpb, k1 = min(nk, k0 + kpb);
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kStages; i++) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        mbar_init(&tfull, 1);
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(&taddr_s, NE <= 128 ? 128 : 256);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = taddr_s;
+
+    if (warp == 0 && lane == 0) {
+        for (int kc = k0, it = 0; kc < k1; kc++, it++) {
+            const int s = it % kStages;
+            if (it >= kStages) mbar_wait(&empty[s], (uint32_t)((it / kStages) - 1) & 1u, status, lim);
+            unsigned char* st = smem + (size_t)s * kStage;
+            mbar_arrive_expect_tx(&full[s], kStage);
+            tma_load_2d(st, &map_x, kc * 64, m0, &full[s]);
+            tma_load_2d(st + kTileBytesA, &map_wr, kc * 64, 0, &full[s]);
+        }
+    } else if (warp == 1 && lane == 0) {
+        constexpr uint32_t idesc = idesc_bf16_m128(NE);
+        for (int kc = k0, it = 0; kc < k1; kc++, it++) {
+            const int s = it % kStages;
+            mbar_wait(&full[s], (uint32_t)(it / kStages) & 1u, status, lim);
+            tc_fence_after();
+            unsigned char* st = smem + (size_t)s * kStage;
+            umma_k64(tmem, st, st + kTileBytesA, idesc, it > 0);
+            umma_commit(&empty[s]);
+        }
+        umma_commit(&tfull);
+    } else if (warp >= 2) {
+        const int q = warp & 3;
+        const int row = 32 * q + lane;
+        const int t = m0 + row;
+        mbar_wait(&tfull, 0, status, lim);
+        tc_fence_after();
+        float* dst = part + ((size_t)split * T + t) * E;
+#pragma unroll 1
+        for (int c = 0; c < NE; c += 32) {
+            uint32_t r[32];
+            tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)c, r);
+            tmem_ld_wait();
+            if (t < T && k1 > k0)
+#pragma unroll
+                for (int i = 0; i < 32; i++)
+                    if (c + i < E) dst[c + i] = __uint_as_float(r[i]);
+            if (t < T && k1 <= k0)
+                for (int i = 0; i < 32; i++)
+                    if (c + i < E) dst[c + i] = 0.0f;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) tmem_dealloc(tmem, NE <= 128 ? 128 : 256);
+}
+
+// ================================================================= selection
+// Selection from K-split partial logits (summed in split order).
+template <int S>
+__global__ void __launch_bounds__(256) select_part_kernel(const float* __restrict__ part, int nsplit, int T, int E,
+                                                          float p, int rule, int gate, int32_t* ids, int32_t* counts,
+                                                          float* gates, float* logits_out, unsigned* status) {
+    const int lane = threadIdx.x & 31;
+    const int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (t >= T) return;
+    auto load = [&](int j) {
+        float v = 0.0f;
+        for (int s = 0; s < nsplit; s++) v += part[((size_t)s * T + t) * E + j];
+        return v;
+    };
+    unsigned long long key[S];
+    bool finite = true;
+    const int k = warp_select<S>(load, E, p, rule, key, &finite);
+    if (!finite && lane == 0) record_status(status, PP_ERR_NONFINITE);
+#pragma unroll
+    for (int s = 0; s < S; s++) {
+        const int r = lane * S + s;
+        if (r >= E) continue;
+        const bool on = finite && r < k;
+        ids[(size_t)t * E + r] = on ? key_index(key[s]) : -1;
+        gates[(size_t)t * E + r] = on ? gate_of(gate, key[s]) : 0.0f;
+    }
+    if (lane == 0) counts[t] = k;
+    if (logits_out)
+        for (int j = lane; j < E; j += 32) logits_out[(size_t)t * E + j] = load(j);
+}
+
+__global__ void __launch_bounds__(256) select_part_cta_kernel(const float* __restrict__ part, int nsplit, int T,
+                                                              int E, float p, int rule, int gate, int32_t* ids,
+                                                              int32_t* counts, float* gates, float* logits_out,
+                                                              unsigned* status) {
+    __shared__ __align__(16) CtaSelScratch sc;
+    const int t = blockIdx.x;
+    auto load = [&](int j) {
+        float v = 0.0f;
+        for (int s = 0; s < nsplit; s++) v += part[((size_t)s * T + t) * E + j];
+        return v;
+    };
+    bool on;
+    int r;
+    float g;
+    const int k = cta_select_fn(load, E, p, rule, sc, status, &on, &r, &g);
+    const int j = threadIdx.x;
+    if (j < E) {
+        ids[(size_t)t * E + r] = on ? j : -1;
+        gates[(size_t)t * E + r] = on ? (gate == PP_GATE_NONE ? 1.0f : sigmoidf_(g)) : 0.0f;
+        if (logits_out) logits_out[(size_t)t * E + j] = g;
+    }
+    if (j == 0) counts[t] = k;
+}
+
+// ================================================================== dispatch
+// bits[t][w]: bit (e % 32) of word e / 32 set when token t activated e;
+// gexp[t][e]: the gate weight of that assignment (gates of a repeated id
+// add up), 0 where e is not activated.  Invalid ids and counts are recorded
+// and skipped.
+__global__ void dispatch_bits_kernel(const int32_t* __restrict__ ids, const int32_t* __restrict__ counts,
+                                     const float* __restrict__ gates, int T, int E, uint32_t* bits, float* gexp,
+                                     unsigned* status) {
+    const int t = blockIdx.x * blockDim.x + threadIdx.x;
+    if (t >= T) return;
+    uint32_t w[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    float* grow = gexp + (size_t)t * E;
+    for (int e = 0; e < E; e++) grow[e] = 0.0f;
+    int k = counts[t];
+    if (k < 0 || k > E) {
+        record_status(status, PP_ERR_INVALID_ARG);
+        k = k < 0 ? 0 : E;
+    }
+    for (int r = 0; r < k; r++) {
+        const int e = ids[(size_t)t * E + r];
+        if (e < 0 || e >= E) {
+            record_status(status, PP_ERR_INVALID_ARG);
+            continue;
+        }
+        w[e >> 5] |= 1u << (e & 31);
+        grow[e] += gates[(size_t)t * E + r];
+    }
+#pragma unroll
+    for (int i = 0; i < 8; i++) bits[(size_t)t * 8 + i] = w[i];
+}
+
+// Token block b (256 tokens, one per thread): per-warp counts of every
+// expert via ballots; block totals blkcnt[b][e].
+constexpr int kDispBlock = 256;
+
+__global__ void __launch_bounds__(kDispBlock) dispatch_count_kernel(const uint32_t* __restrict__ bits, int T, int E,
+                                                                    int* wcnt, int* blkcnt) {
+    const int b = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int t = b * kDispBlock + threadIdx.x;
+    uint32_t w[8];
+#pragma unroll
+    for (int i = 0; i < 8; i++) w[i] = t < T ? bits[(size_t)t * 8 + i] : 0u;
+    __shared__ int sc[8][kMaxExperts];
+    for (int e = 0; e < E; e++) {
+        const unsigned bal = __ballot_sync(kFull, (w[e >> 5] >> (e & 31)) & 1u);
+        if (lane == 0) sc[warp][e] = __popc(bal);
+    }
+    __syncthreads();
+    for (int e = threadIdx.x; e < E; e += kDispBlock) {
+        int s = 0;
+        for (int v = 0; v < 8; v++) {
+            wcnt[((size_t)b * 8 + v) * E + e] = s;  // exclusive prefix over the block's warps
+            s += sc[v][e];
+        }
+        blkcnt[(size_t)b * E + e] = s;
+    }
+}
+
+// One block, thread e: hist, offsets (exclusive scan over experts), the
+// per-token-block bases and the expert's 128-row work items.
+__global__ void __launch_bounds__(kMaxExperts) dispatch_scan_kernel(const int* __restrict__ blkcnt, int nblk, int E,
+                                                                    int* offsets, int* blkbase, WorkItem* items,
+                                                                    int* n_items) {
+    const int e = threadIdx.x;
+    __shared__ int sh[kMaxExperts], si[kMaxExperts];
+    int h = 0;
+    if (e < E)
+        for (int b = 0; b < nblk; b++) h += blkcnt[(size_t)b * E + e];
+    sh[e] = e < E ? h : 0;
+    si[e] = e < E ? (h + 127) / 128 : 0;
+    __syncthreads();
+    if (e == 0) {  // exclusive scans of counts and item counts (E <= 256)
+        int a = 0, n = 0;
+        for (int i = 0; i < E; i++) {
+            const int c = sh[i], m = si[i];
+            sh[i] = a;
+            si[i] = n;
+            a += c;
+            n += m;
+        }
+        offsets[E] = a;
+        *n_items = n;
+    }
+    __syncthreads();
+    if (e >= E) return;
+    const int off = sh[e];
+    offsets[e] = off;
+    int base = off;
+    for (int b = 0; b < nblk; b++) {
+        blkbase[(size_t)b * E + e] = base;
+        base += blkcnt[(size_t)b * E + e];
+    }
+    int n = si[e];
+    for (int m = 0; m < h; m += 128) items[n++] = WorkItem{e, off + m, min(128, h - m), 0};
+}
+
+// Token block b again: each token writes itself (and its gate weight) at
+// base + (earlier warps) + (earlier lanes) for every activated expert, so
+// tokens stay in ascending order within each expert; invpos[t][e] records
+// where (t, e) landed.
+__global__ void __launch_bounds__(kDispBlock) dispatch_scatter_kernel(const uint32_t* __restrict__ bits,
+                                                                      const float* __restrict__ gexp, int T, int E,
+                                                                      const int* __restrict__ wcnt,
+                                                                      const int* __restrict__ blkbase,
+                                                                      int* perm_token, float* perm_gate,
+                                                                      int* invpos) {
+    const int b = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int t = b * kDispBlock + threadIdx.x;
+    const bool live = t < T;
+    uint32_t w[8];
+#pragma unroll
+    for (int i = 0; i < 8; i++) w[i] = live ? bits[(size_t)t * 8 + i] : 0u;
+    const unsigned lt = (1u << lane) - 1u;
+    for (int e = 0; e < E; e++) {
+        const bool on = (w[e >> 5] >> (e & 31)) & 1u;
+        const unsigned bal = __ballot_sync(kFull, on);
+        if (on) {
+            const int pos = blkbase[(size_t)b * E + e] + wcnt[((size_t)b * 8 + warp) * E + e] + __popc(bal & lt);
+            perm_token[pos] = t;
+            perm_gate[pos] = gexp[(size_t)t * E + e];
+            invpos[(size_t)t * E + e] = pos;
+        }
+    }
+}
+
+// =============================================================== grouped G/U
+// Persistent over work items.  NB = 128 (SwiGLU: gate rows then up rows) or
+// 64 (non-gated: up rows).  Two TMEM accumulators let the epilogue of one
+// item overlap the MMAs of the next.
+template <int NB>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    gu_gemm_kernel(const __grid_constant__ CUtensorMap map_x1, const __grid_constant__ CUtensorMap map_wg,
+                   const __grid_constant__ CUtensorMap map_wu, const WorkItem* __restrict__ items,
+                   const int* __restrict__ n_items_p, const int* __restrict__ perm_token,
+                   const float* __restrict__ perm_gate, int nk, int act, __nv_bfloat16* H, unsigned* status,
+                   uint64_t lim) {
+    constexpr int kStages = NB == 128 ? 6 : 8;
+    constexpr int kTileB = NB * 128;
+    constexpr int kStage = kTileBytesA + kTileB;
+    constexpr uint32_t kCols = 2 * NB;  // two accumulators
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    __shared__ uint64_t full[kStages], empty[kStages], tfull[2], tempty[2];
+    __shared__ uint32_t taddr_s;
+    __shared__ int rows_s[128];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n_items = *n_items_p;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kStages; i++) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        for (int i = 0; i < 2; i++) {
+            mbar_init(&tfull[i], 1);
+            mbar_init(&tempty[i], 4);
+        }
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(&taddr_s, kCols < 32 ? 32 : kCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = taddr_s;
+
+    if (warp == 0) {
+        int it = 0;
+        for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x) {
+            const WorkItem w = items[wi];
+            // the item's token rows (padding rows repeat the last token)
+            for (int i = lane; i < 128; i += 32) rows_s[i] = perm_token[w.a0 + min(i, w.cnt - 1)];
+            __syncwarp();
+            // only the item's live rows are gathered (lane g issues group g);
+            // padding rows keep stale data and only feed accumulator rows the
+            // epilogue never stores
+            const int ng = (w.cnt + 3) >> 2;
+            const int r0 = lane < ng ? rows_s[4 * lane] : 0, r1 = lane < ng ? rows_s[4 * lane + 1] : 0;
+            const int r2 = lane < ng ? rows_s[4 * lane + 2] : 0, r3 = lane < ng ? rows_s[4 * lane + 3] : 0;
+            for (int kc = 0; kc < nk; kc++, it++) {
+                const int s = it % kStages;
+                unsigned char* st = smem + (size_t)s * kStage;
+                if (lane == 0) {
+                    if (it >= kStages) mbar_wait(&empty[s], (uint32_t)((it / kStages) - 1) & 1u, status, lim);
+                    mbar_arrive_expect_tx(&full[s], (uint32_t)(ng * 512 + kTileB));
+                }
+                __syncwarp();
+                if (lane < ng) tma_gather4(st + lane * 512, &map_x1, kc * 64, r0, r1, r2, r3, &full[s]);
+                if (lane == 0) {
+                    if (NB == 128) {
+                        tma_load_2d(st + kTileBytesA, &map_wg, kc * 64, w.e * 64, &full[s]);
+                        tma_load_2d(st + kTileBytesA + 64 * 128, &map_wu, kc * 64, w.e * 64, &full[s]);
+                    } else {
+                        tma_load_2d(st + kTileBytesA, &map_wu, kc * 64, w.e * 64, &full[s]);
+                    }
+                }
+            }
+            __syncwarp();
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16_m128(NB);
+            int it = 0, acc = 0;
+            for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x, acc++) {
+                const int a = acc & 1;
+                if (acc >= 2) mbar_wait(&tempty[a], (uint32_t)((acc >> 1) - 1) & 1u, status, lim);
+                tc_fence_after();
+                for (int kc = 0; kc < nk; kc++, it++) {
+                    const int s = it % kStages;
+                    mbar_wait(&full[s], (uint32_t)(it / kStages) & 1u, status, lim);
+                    tc_fence_after();
+                    unsigned char* st = smem + (size_t)s * kStage;
+                    umma_k64(tmem + (uint32_t)(a * NB), st, st + kTileBytesA, idesc, kc > 0);
+                    umma_commit(&empty[s]);
+                }
+                umma_commit(&tfull[a]);
+            }
+        }
+        __syncwarp();
+    } else {
+        const int q = warp & 3;
+        const int row = 32 * q + lane;
+        int acc = 0;
+        for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x, acc++) {
+            const WorkItem w = items[wi];
+            const int a = acc & 1;
+            mbar_wait(&tfull[a], (uint32_t)(acc >> 1) & 1u, status, lim);
+            tc_fence_after();
+            const bool live = row < w.cnt;
+            const float gw = live ? perm_gate[w.a0 + row] : 0.0f;
+            const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(a * NB);
+#pragma unroll 1
+            for (int c = 0; c < 64; c += 32) {
+                uint32_t u[32];
+                tmem_ld32(base + (uint32_t)(NB == 128 ? 64 + c : c), u);
+                float h[32];
+                if (NB == 128) {
+                    uint32_t g[32];
+                    tmem_ld32(base + (uint32_t)c, g);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < 32; i++) h[i] = act_h(PP_ACT_SWIGLU, __uint_as_float(u[i]), __uint_as_float(g[i])) * gw;
+                } else {
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < 32; i++) h[i] = act_h(act, __uint_as_float(u[i]), 0.0f) * gw;
+                }
+                if (live) {
+                    uint4* dst = reinterpret_cast<uint4*>(H + (size_t)(w.a0 + row) * 64 + c);
+#pragma unroll
+                    for (int v = 0; v < 4; v++)
+                        dst[v] = make_uint4(pack_bf16x2(h[8 * v], h[8 * v + 1]), pack_bf16x2(h[8 * v + 2], h[8 * v + 3]),
+                                            pack_bf16x2(h[8 * v + 4], h[8 * v + 5]), pack_bf16x2(h[8 * v + 6], h[8 * v + 7]));
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[a]);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) tmem_dealloc(tmem, kCols < 32 ? 32 : kCols);
+}
+
+PP_DEVINL bool jt_first_overflow(const WorkItem& w, long long ycap) { return (long long)w.a0 + w.cnt > ycap; }
+
+// ============================================================== grouped down
+// Persistent over work items; per item the H tile is loaded once and the
+// njt 256-wide slices of d stream through the B ring.  Two 256-column TMEM
+// accumulators overlap the reduction epilogue with the next slice's MMAs.
+__global__ void __launch_bounds__(kTcThreads, 1)
+    down_gemm_kernel(const __grid_constant__ CUtensorMap map_h, const __grid_constant__ CUtensorMap map_wd,
+                     const WorkItem* __restrict__ items, const int* __restrict__ n_items_p,
+                     const int* __restrict__ perm_token, int d, int njt, __nv_bfloat16* Y, long long ycap,
+                     float* yacc, int* overflow, unsigned* status, uint64_t lim) {
+    constexpr int kStages = 4;
+    constexpr int kTileB = 256 * 128;
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    unsigned char* tileA = smem;
+    unsigned char* ringB = smem + kTileBytesA;
+    __shared__ uint64_t full[kStages], empty[kStages], tfull[2], tempty[2], afull, aempty;
+    __shared__ uint32_t taddr_s;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n_items = *n_items_p;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kStages; i++) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        for (int i = 0; i < 2; i++) {
+            mbar_init(&tfull[i], 1);
+            mbar_init(&tempty[i], 4);
+        }
+        mbar_init(&afull, 1);
+        mbar_init(&aempty, 1);
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(&taddr_s, 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = taddr_s;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int it = 0, ii = 0;
+            for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x, ii++) {
+                const WorkItem w = items[wi];
+                if (ii >= 1) mbar_wait(&aempty, (uint32_t)(ii - 1) & 1u, status, lim);
+                mbar_arrive_expect_tx(&afull, kTileBytesA);
+                tma_load_2d(tileA, &map_h, 0, w.a0, &afull);
+                for (int jt = 0; jt < njt; jt++, it++) {
+                    const int s = it % kStages;
+                    if (it >= kStages) mbar_wait(&empty[s], (uint32_t)((it / kStages) - 1) & 1u, status, lim);
+                    mbar_arrive_expect_tx(&full[s], kTileB);
+                    tma_load_2d(ringB + (size_t)s * kTileB, &map_wd, w.e * 64, jt * 256, &full[s]);
+                }
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16_m128(256);
+            int it = 0, acc = 0, ii = 0;
+            for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x, ii++) {
+                mbar_wait(&afull, (uint32_t)ii & 1u, status, lim);
+                for (int jt = 0; jt < njt; jt++, it++, acc++) {
+                    const int a = acc & 1;
+                    if (acc >= 2) mbar_wait(&tempty[a], (uint32_t)((acc >> 1) - 1) & 1u, status, lim);
+                    const int s = it % kStages;
+                    mbar_wait(&full[s], (uint32_t)(it / kStages) & 1u, status, lim);
+                    tc_fence_after();
+                    umma_k64(tmem + (uint32_t)(a * 256), tileA, ringB + (size_t)s * kTileB, idesc, false);
+                    umma_commit(&empty[s]);
+                    umma_commit(&tfull[a]);
+                }
+                umma_commit(&aempty);
+            }
+        }
+        __syncwarp();
+    } else {
+        const int q = warp & 3;
+        const int row = 32 * q + lane;
+        int acc = 0;
+        for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x) {
+            const WorkItem w = items[wi];
+            const bool live = row < w.cnt;
+            const long long arow = (long long)w.a0 + row;
+            const bool in_buf = live && arow < ycap;
+            const int tok = live && !in_buf ? perm_token[arow] : -1;
+            float* yrow = tok >= 0 ? yacc + (size_t)tok * d : nullptr;
+            if (tok >= 0 && jt_first_overflow(w, ycap)) *overflow = 1;
+            __nv_bfloat16* Yrow = in_buf ? Y + (size_t)arow * d : nullptr;
+            for (int jt = 0; jt < njt; jt++, acc++) {
+                const int a = acc & 1;
+                mbar_wait(&tfull[a], (uint32_t)(acc >> 1) & 1u, status, lim);
+                tc_fence_after();
+                const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(a * 256);
+#pragma unroll 1
+                for (int c = 0; c < 256; c += 32) {
+                    uint32_t r[32];
+                    tmem_ld32(base + (uint32_t)c, r);
+                    tmem_ld_wait();
+                    const int j0 = jt * 256 + c;
+                    if (Yrow) {
+#pragma unroll
+                        for (int v = 0; v < 4; v++)
+                            if (j0 + 8 * v < d)
+                                *reinterpret_cast<uint4*>(Yrow + j0 + 8 * v) = make_uint4(
+                                    pack_bf16x2(__uint_as_float(r[8 * v]), __uint_as_float(r[8 * v + 1])),
+                                    pack_bf16x2(__uint_as_float(r[8 * v + 2]), __uint_as_float(r[8 * v + 3])),
+                                    pack_bf16x2(__uint_as_float(r[8 * v + 4]), __uint_as_float(r[8 * v + 5])),
+                                    pack_bf16x2(__uint_as_float(r[8 * v + 6]), __uint_as_float(r[8 * v + 7])));
+                    } else if (yrow) {
+#pragma unroll
+                        for (int v = 0; v < 8; v++)
+                            if (j0 + 4 * v < d)
+                                red_add_v4(yrow + j0 + 4 * v, __uint_as_float(r[4 * v]), __uint_as_float(r[4 * v + 1]),
+                                           __uint_as_float(r[4 * v + 2]), __uint_as_float(r[4 * v + 3]));
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&tempty[a]);
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) tmem_dealloc(tmem, 512);
+}
+
+// =================================================================== combine
+// One CTA per token: y[t] = (accumulator row, if any overflow) + the rows of
+// t's assignments in ascending expert order; fp32 sums, output bf16.
+__global__ void __launch_bounds__(128) combine_kernel(const uint32_t* __restrict__ bits, const int* __restrict__ invpos,
+                                                      const __nv_bfloat16* __restrict__ Y, long long ycap,
+                                                      float* yacc, const int* __restrict__ overflow, int T, int E,
+                                                      int d, __nv_bfloat16* y) {
+    const int t = blockIdx.x;
+    __shared__ int pos_s[kMaxExperts];
+    __shared__ int n_s;
+    if (threadIdx.x == 0) {
+        int n = 0;
+        for (int wdx = 0; wdx < 8; wdx++) {
+            uint32_t w = bits[(size_t)t * 8 + wdx];
+            while (w) {
+                const int e = wdx * 32 + __ffs(w) - 1;
+                w &= w - 1;
+                const int pos = invpos[(size_t)t * E + e];
+                if (pos < ycap) pos_s[n++] = pos;
+            }
+        }
+        n_s = n;
+    }
+    __syncthreads();
+    const int n = n_s;
+    const bool ovf = *overflow != 0;
+    for (int c = threadIdx.x * 8; c < d; c += blockDim.x * 8) {
+        float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+        if (ovf) {
+            float4* ya = reinterpret_cast<float4*>(yacc + (size_t)t * d + c);
+            const float4 a0 = ya[0], a1 = ya[1];
+            acc[0] = a0.x; acc[1] = a0.y; acc[2] = a0.z; acc[3] = a0.w;
+            acc[4] = a1.x; acc[5] = a1.y; acc[6] = a1.z; acc[7] = a1.w;
+            ya[0] = make_float4(0.f, 0.f, 0.f, 0.f);  // keep the accumulator zero at rest
+            ya[1] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        for (int i = 0; i < n; i++) {
+            const uint4 v = *reinterpret_cast<const uint4*>(Y + (size_t)pos_s[i] * d + c);
+            acc[0] += bf16lo(v.x); acc[1] += bf16hi(v.x); acc[2] += bf16lo(v.y); acc[3] += bf16hi(v.y);
+            acc[4] += bf16lo(v.z); acc[5] += bf16hi(v.z); acc[6] += bf16lo(v.w); acc[7] += bf16hi(v.w);
+        }
+        *reinterpret_cast<uint4*>(y + (size_t)t * d + c) =
+            make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]), pack_bf16x2(acc[4], acc[5]),
+                       pack_bf16x2(acc[6], acc[7]));
+    }
+}
+
+// ====================================================================== host
+namespace {
+
+bool encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer, uint32_t box_inner,
+               uint32_t box_outer) {
+    auto enc = tensor_map_encoder();
+    if (!enc) return false;
+    const cuuint64_t dims[2] = {inner, outer};
+    const cuuint64_t strides[1] = {inner * 2};
+    const cuuint32_t box[2] = {box_inner, box_outer};
+    const cuuint32_t estr[2] = {1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <typename K>
+cudaError_t set_smem(K kern, size_t bytes) {
+    return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+}
+
+int router_ne(int E) { return E <= 32 ? 32 : E <= 64 ? 64 : E <= 128 ? 128 : E <= 160 ? 160 : E <= 192 ? 192 : E <= 224 ? 224 : 256; }
+
+template <int NE>
+cudaError_t launch_router(const CUtensorMap& mx, const CUtensorMap& mwr, int T, int E, int nk, int kpb, int nsplit,
+                          float* part, unsigned* status, uint64_t lim, cudaStream_t st) {
+    const size_t smem = 4 * (size_t)(kTileBytesA + NE * 128) + 1024;
+    cudaError_t e = set_smem(router_gemm_kernel<NE>, smem);
+    if (e != cudaSuccess) return e;
+    router_gemm_kernel<NE><<<dim3((T + 127) / 128, nsplit), kTcThreads, smem, st>>>(mx, mwr, T, E, nk, kpb, part,
+                                                                                     status, lim);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+GroupedPlan grouped_plan(int T, int d, int E, int sms) {
+    GroupedPlan g{};
+    g.nk = (d + 63) / 64;  // the last chunk's columns past d are zero-filled by TMA
+    // router K splits: at most one wave of CTAs, at least 4 chunks each
+    const int mt = (T + 127) / 128;
+    const int ns = std::max(1, std::min(sms / mt, std::min(g.nk / 4, 64)));
+    g.kpb = (g.nk + ns - 1) / ns;
+    g.nsplit = (g.nk + g.kpb - 1) / g.kpb;
+    g.max_items = (int)std::min<long long>((long long)T * E / 128 + E + 1, (long long)T * E);
+    g.nnz_max = (long long)T * E;
+    g.ycap = (long long)T * std::min(E, 64);  // assignment rows kept for the combine
+    return g;
+}
+
+cudaError_t grouped_route(const GroupedArgs& a, cudaStream_t st) {
+    const GroupedPlan& g = a.plan;
+    CUtensorMap mx, mwr;
+    const int NE = router_ne(a.E);
+    if (!encode_2d(&mx, a.x, a.d, a.T, 64, 128) || !encode_2d(&mwr, a.Wr, a.d, a.E, 64, NE)) return cudaErrorInvalidValue;
+    cudaError_t e;
+    switch (NE) {
+        case 32: e = launch_router<32>(mx, mwr, a.T, a.E, g.nk, g.kpb, g.nsplit, a.part, a.status, a.timeout_ns, st); break;
+        case 64: e = launch_router<64>(mx, mwr, a.T, a.E, g.nk, g.kpb, g.nsplit, a.part, a.status, a.timeout_ns, st); break;
+        case 128: e = launch_router<128>(mx, mwr, a.T, a.E, g.nk, g.kpb, g.nsplit, a.part, a.status, a.timeout_ns, st); break;
+        case 160: e = launch_router<160>(mx, mwr, a.T, a.E, g.nk, g.kpb, g.nsplit, a.part, a.status, a.timeout_ns, st); break;
+        case 192: e = launch_router<192>(mx, mwr, a.T, a.E, g.nk, g.kpb, g.nsplit, a.part, a.status, a.timeout_ns, st); break;
+        case 224: e = launch_router<224>(mx, mwr, a.T, a.E, g.nk, g.kpb, g.nsplit, a.part, a.status, a.timeout_ns, st); break;
+        default: e = launch_router<256>(mx, mwr, a.T, a.E, g.nk, g.kpb, g.nsplit, a.part, a.status, a.timeout_ns, st); break;
+    }
+    if (e != cudaSuccess) return e;
+    if (a.T <= 64) {
+        select_part_cta_kernel<<<a.T, 256, 0, st>>>(a.part, g.nsplit, a.T, a.E, a.p, a.rule, a.gate, a.ids, a.counts,
+                                                    a.gates, a.logits_out, a.status);
+        return cudaGetLastError();
+    }
+    const dim3 grid((a.T + 7) / 8), block(256);
+    switch (sel_slots_for(a.E)) {
+        case 1: select_part_kernel<1><<<grid, block, 0, st>>>(a.part, g.nsplit, a.T, a.E, a.p, a.rule, a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status); break;
+        case 2: select_part_kernel<2><<<grid, block, 0, st>>>(a.part, g.nsplit, a.T, a.E, a.p, a.rule, a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status); break;
+        case 4: select_part_kernel<4><<<grid, block, 0, st>>>(a.part, g.nsplit, a.T, a.E, a.p, a.rule, a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status); break;
+        default: select_part_kernel<8><<<grid, block, 0, st>>>(a.part, g.nsplit, a.T, a.E, a.p, a.rule, a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status); break;
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
+    const GroupedPlan& g = a.plan;
+    const bool gated = a.act == PP_ACT_SWIGLU;
+    cudaError_t e;
+    // dispatch
+    const int nblk = (a.T + kDispBlock - 1) / kDispBlock;
+    dispatch_bits_kernel<<<(a.T + 255) / 256, 256, 0, st>>>(a.ids, a.counts, a.gates, a.T, a.E, a.bits, a.gexp,
+                                                             a.status);
+    dispatch_count_kernel<<<nblk, kDispBlock, 0, st>>>(a.bits, a.T, a.E, a.wcnt, a.blkcnt);
+    dispatch_scan_kernel<<<1, kMaxExperts, 0, st>>>(a.blkcnt, nblk, a.E, a.offsets, a.blkbase,
+                                                   reinterpret_cast<WorkItem*>(a.items), a.n_items);
+    dispatch_scatter_kernel<<<nblk, kDispBlock, 0, st>>>(a.bits, a.gexp, a.T, a.E, a.wcnt, a.blkbase, a.perm_token,
+                                                        a.perm_gate, a.invpos);
+    if ((e = cudaMemsetAsync(a.overflow, 0, 4, st)) != cudaSuccess) return e;
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    // grouped gate/up
+    CUtensorMap mx1, mwg, mwu, mh, mwd;
+    if (!encode_2d(&mx1, a.x, a.d, a.T, 64, 1) || !encode_2d(&mwu, a.Wu, a.d, (uint64_t)a.E * 64, 64, 64) ||
+        !encode_2d(&mwg, gated ? a.Wg : a.Wu, a.d, (uint64_t)a.E * 64, 64, 64) ||
+        !encode_2d(&mh, a.H, 64, (uint64_t)g.nnz_max + 128, 64, 128) ||
+        !encode_2d(&mwd, a.Wd, (uint64_t)a.E * 64, a.d, 64, 256))
+        return cudaErrorInvalidValue;
+    const int grid = std::max(1, std::min(sms, g.max_items));
+    const WorkItem* items = reinterpret_cast<const WorkItem*>(a.items);
+    if (gated) {
+        const size_t smem = 6 * (size_t)(kTileBytesA + 128 * 128) + 1024;
+        if ((e = set_smem(gu_gemm_kernel<128>, smem)) != cudaSuccess) return e;
+        gu_gemm_kernel<128><<<grid, kTcThreads, smem, st>>>(mx1, mwg, mwu, items, a.n_items, a.perm_token, a.perm_gate,
+                                                            g.nk, a.act, a.H, a.status, a.timeout_ns);
+    } else {
+        const size_t smem = 8 * (size_t)(kTileBytesA + 64 * 128) + 1024;
+        if ((e = set_smem(gu_gemm_kernel<64>, smem)) != cudaSuccess) return e;
+        gu_gemm_kernel<64><<<grid, kTcThreads, smem, st>>>(mx1, mwg, mwu, items, a.n_items, a.perm_token, a.perm_gate,
+                                                           g.nk, a.act, a.H, a.status, a.timeout_ns);
+    }
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    // grouped down + scatter-add
+    {
+        const size_t smem = (size_t)kTileBytesA + 4 * (size_t)256 * 128 + 1024;
+        if ((e = set_smem(down_gemm_kernel, smem)) != cudaSuccess) return e;
+        down_gemm_kernel<<<grid, kTcThreads, smem, st>>>(mh, mwd, items, a.n_items, a.perm_token, a.d,
+                                                         (a.d + 255) / 256, a.Y, g.ycap, a.yacc, a.overflow,
+                                                         a.status, a.timeout_ns);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    combine_kernel<<<a.T, 128, 0, st>>>(a.bits, a.invpos, a.Y, g.ycap, a.yacc, a.overflow, a.T, a.E, a.d,
+                                        reinterpret_cast<__nv_bfloat16*>(a.y));
+    return cudaGetLastError();
+}
+
+}  // namespace pp

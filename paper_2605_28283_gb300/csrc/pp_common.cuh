@@ -74,16 +74,20 @@ PP_DEVINL bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Wait for the phase with the given parity to complete, for at most
-// limit_ns.  On expiry records PP_ERR_TIMEOUT and returns false.
+// limit_ns.  On expiry records PP_ERR_TIMEOUT and returns false.  A wait
+// that has lasted over 1 ms also gives up as soon as another wait has
+// recorded an error, so one failure cannot chain into many full timeouts.
 PP_DEVINL bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned* status, uint64_t limit_ns) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     while (true) {
         if (mbar_try_wait(bar, parity)) return true;
-        if (globaltimer_ns() - t0 > limit_ns) {
+        const uint64_t dt = globaltimer_ns() - t0;
+        if (dt > limit_ns) {
             record_status(status, PP_ERR_TIMEOUT);
             return false;
         }
+        if (dt > 1000000ull && *reinterpret_cast<volatile unsigned*>(status) != 0u) return false;
     }
 }
 

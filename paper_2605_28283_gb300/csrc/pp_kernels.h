@@ -8,6 +8,8 @@
 
 #include <algorithm>
 
+#include <cuda_bf16.h>
+
 #include "prunepath.h"
 
 namespace pp {
@@ -63,6 +65,60 @@ cudaError_t select_launch(const float* logits, int T, int E, float p, int rule, 
 cudaError_t stats_launch(const int32_t* counts, int T, int E, uint64_t* acc, cudaStream_t st);
 cudaError_t wait_timeout_launch(unsigned* flag, unsigned* status, long long timeout_ns,
                                 cudaStream_t st);
+
+// ------------------------------------------------- tensor-core grouped path
+struct GroupedPlan {
+    int nk;          // 64-wide K chunks of d
+    int kpb;         // router K chunks per split
+    int nsplit;      // router K splits
+    int max_items;   // upper bound on 128-row work items
+    long long nnz_max;  // upper bound on (token, expert) assignments
+    long long ycap;     // rows of the bf16 assignment-output buffer
+};
+
+struct GroupedArgs {
+    GroupedPlan plan;
+    const void* x;
+    const void* Wr;
+    const void* Wg;
+    const void* Wu;
+    const void* Wd;
+    void* y;
+    int T, d, E, act, gate, rule;
+    float p;
+    int32_t* ids;
+    int32_t* counts;
+    float* gates;
+    float* logits_out;  // optional final logits
+    float* part;        // [nsplit][T][E] router partials
+    uint32_t* bits;     // [T][8]
+    float* gexp;        // [T][E] gate weight per (token, expert)
+    int* invpos;        // [T][E] permuted row of (token, expert)
+    int* wcnt;          // [T/256][8][E] per-warp exclusive counts
+    int* blkcnt;        // [T/256][E]
+    int* blkbase;       // [T/256][E]
+    int* offsets;       // [E + 1]
+    void* items;        // [max_items] work items
+    int* n_items;
+    int* perm_token;    // [nnz_max]
+    float* perm_gate;   // [nnz_max]
+    __nv_bfloat16* H;   // [nnz_max + 128][64]
+    __nv_bfloat16* Y;   // [ycap][d] assignment outputs
+    float* yacc;        // [T][d] overflow accumulator, zero at rest
+    int* overflow;      // set when any assignment went to yacc
+    unsigned* status;
+    uint64_t timeout_ns;
+};
+
+GroupedPlan grouped_plan(int T, int d, int E, int sms);
+cudaError_t grouped_route(const GroupedArgs& a, cudaStream_t st);
+cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st);
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point (nullptr if unavailable)
+typedef CUresult (*TensorMapEncodeFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                      const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                      CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+TensorMapEncodeFn tensor_map_encoder();
 
 inline int sel_slots_for(int E) { return E <= 32 ? 1 : E <= 64 ? 2 : E <= 128 ? 4 : 8; }
 

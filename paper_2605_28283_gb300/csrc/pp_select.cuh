@@ -188,13 +188,13 @@ PP_DEVINL long long prefix_threshold(float p, unsigned long long Z) {
 // Returns the activated count (CTA-uniform).  On return: *sel = whether
 // expert j (= threadIdx.x) is activated, *rank = its rank (valid j only),
 // *gval = its logit.  All threads of the CTA must call it.
-PP_DEVINL int cta_select(const float* __restrict__ logits_row, int E, float p, int rule,
-                         CtaSelScratch& sc, unsigned* status, bool* sel, int* rank,
-                         float* gval) {
+template <typename Load>
+PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, CtaSelScratch& sc, unsigned* status,
+                            bool* sel, int* rank, float* gval) {
     const int j = threadIdx.x;
     const int lane = j & 31, warp = j >> 5, nwarps = blockDim.x >> 5;
     const bool valid = j < E;
-    const float g = valid ? __ldcg(logits_row + j) : -INFINITY;
+    const float g = valid ? load(j) : -INFINITY;
     *gval = g;
     const bool fin = !valid || isfinite(g);
     if (!__syncthreads_and(fin)) {
@@ -267,6 +267,12 @@ PP_DEVINL int cta_select(const float* __restrict__ logits_row, int E, float p, i
     *rank = r;
     const int k = __syncthreads_count(on);
     return k;
+}
+
+// Same, reading the logits (written by other CTAs earlier) from a row.
+PP_DEVINL int cta_select(const float* __restrict__ logits_row, int E, float p, int rule, CtaSelScratch& sc,
+                         unsigned* status, bool* sel, int* rank, float* gval) {
+    return cta_select_fn([&](int j) { return __ldcg(logits_row + j); }, E, p, rule, sc, status, sel, rank, gval);
 }
 
 }  // namespace pp
