@@ -139,6 +139,27 @@ pp_status pp_layer(const pp_desc *desc, const void *x, int T, const void *W_r, c
                    const void *W_up, const void *W_down, float p, const pp_selection *sel_out,
                    void *y, void *ws, size_t ws_bytes, void *stream);
 
+/* pp_layer for callers that cannot allocate device memory where they run a
+   layer -- a runtime that has given every byte to its own pool, a loop that
+   must not block on an allocation's implicit synchronisation, a plug-in host
+   that exposes no allocator.  The paper has no counterpart: this entry point
+   exists only for those callers.
+   Same computation and arguments as pp_layer, for T <= 4 tokens and without a
+   workspace.  Its scratch (status word, barrier counter, router logits, gate/up
+   activations: 266,496 bytes) is one static device array that every GPU loading
+   this library keeps until the process exits; no call allocates or frees.
+   - T > 4 (like any shape pp_layer rejects) returns PP_ERR_SHAPE.
+   - The first call on a device, made with that device current, looks up the
+     array's address there; make that first call before any stream capture.
+   - Every call reuses the same array and first clears its status word and
+     barrier counter; calls that overlap on the GPU (other streams, other host
+     threads) race on it, so the caller must serialise them.
+   - status_out (optional, device uint32) receives the call's device-side
+     status (a pp_status code) when the call has run on `stream`. */
+pp_status pp_layer_noalloc(const pp_desc *desc, const void *x, int T, const void *W_r,
+                           const void *W_gate, const void *W_up, const void *W_down, float p,
+                           const pp_selection *sel_out, void *y, uint32_t *status_out, void *stream);
+
 /* FFN-sparsity statistics (Sec. 4.1, s_FFN): adds sum_t counts[t] to
    acc[0] and a histogram of counts (0..E) to acc[1..E+1].  acc is
    [E+2] uint64 on the device, accumulated across calls (one per layer), so
