@@ -99,17 +99,22 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     const int j0 = b * rpc, j1 = min(E, j0 + rpc);
     const int nrows = a.do_route ? max(0, j1 - j0) : 0;
 
-    // x -> shared memory (all T rows are contiguous), and the router rows
-    if (tid == 0) {
+    // The router rows are weights: load them before waiting for the
+    // preceding grid (with programmatic dependent launch this overlaps the
+    // previous layer's tail).  x and the workspace may be that grid's output
+    // or scratch, so they are touched only after the wait.
+    if (tid == 0 && nrows > 0) {
+        const TW* wr = reinterpret_cast<const TW*>(a.Wr);
+        const uint32_t rbytes = (uint32_t)(nrows * rowb);
+        mbar_arrive_expect_tx(&bars[kBarR], rbytes);
+        bulk_g2s(ring4, wr + (size_t)j0 * d, rbytes, &bars[kBarR]);
+    }
+    pdl_wait();
+    pdl_launch_dependents();
+    if (tid == 0) {  // x -> shared memory (all T rows are contiguous)
         const uint32_t bytes = (uint32_t)(T * rowb);
         mbar_arrive_expect_tx(&bars[kBarX], bytes);
         bulk_g2s(xs, a.x, bytes, &bars[kBarX]);
-        if (nrows > 0) {
-            const TW* wr = reinterpret_cast<const TW*>(a.Wr);
-            const uint32_t rbytes = (uint32_t)(nrows * rowb);
-            mbar_arrive_expect_tx(&bars[kBarR], rbytes);
-            bulk_g2s(ring4, wr + (size_t)j0 * d, rbytes, &bars[kBarR]);
-        }
     }
     // every CTA waits for its copy of x here, so no bulk copy is ever still
     // in flight when a CTA that has no work left exits
@@ -178,7 +183,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
                     mask[j] |= 1u << t;
                 }
                 if (publish) {
-                    if (a.sel_ids) {
+                    if (a.sel_ids) {  // ranks are a permutation: every rank slot is written once
                         a.sel_ids[(size_t)t * E + r] = on ? j : -1;
                         a.sel_gates[(size_t)t * E + r] = gv;
                     }
@@ -243,71 +248,124 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     const int nb = (int)(((long long)b * Ntot) / G);
     const int ne = (int)(((long long)(b + 1) * Ntot) / G);
     const int cnt = ne - nb;
-    const bool ph4 = warp < a.NS4 && cnt > warp;
     const uint32_t stage4 = (uint32_t)((gated ? 2 : 1) * rowb);
-    unsigned char* slot4 = ring4 + (size_t)warp * stage4;
-    uint64_t* fb4 = &bars[kBarFull4 + warp];
     const TW* Wg = reinterpret_cast<const TW*>(a.Wg);
     const TW* Wu = reinterpret_cast<const TW*>(a.Wu);
-    auto issue4 = [&](int i) {
+    // neuron i of this CTA (global neuron nb + i) -> ring slot `slot`
+    auto issue4 = [&](int i, int slot) {
         const int q = nb + i;
         const size_t row = (size_t)ulist[q >> 6] * kDExpert + (q & 63);
-        mbar_arrive_expect_tx(fb4, stage4);
+        unsigned char* dst = ring4 + (size_t)slot * stage4;
+        uint64_t* fb = &bars[kBarFull4 + slot];
+        mbar_arrive_expect_tx(fb, stage4);
         if (gated) {
-            bulk_g2s(slot4, Wg + row * d, (uint32_t)rowb, fb4);
-            bulk_g2s(slot4 + rowb, Wu + row * d, (uint32_t)rowb, fb4);
+            bulk_g2s(dst, Wg + row * d, (uint32_t)rowb, fb);
+            bulk_g2s(dst + rowb, Wu + row * d, (uint32_t)rowb, fb);
         } else {
-            bulk_g2s(slot4, Wu + row * d, (uint32_t)rowb, fb4);
+            bulk_g2s(dst, Wu + row * d, (uint32_t)rowb, fb);
         }
     };
+    // dot products of one neuron's gate/up rows (in `slot`) with x over the
+    // 16-byte chunks [c0, c1), per token
+    auto neuron_dots = [&](int slot, int c0, int c1, float (&au)[TS], float (&ag)[TS]) {
+        const unsigned char* base = ring4 + (size_t)slot * stage4;
+        const TW* gs = reinterpret_cast<const TW*>(base);
+        const TW* us = reinterpret_cast<const TW*>(gated ? base + rowb : base);
+#pragma unroll
+        for (int t = 0; t < TS; t++) au[t] = ag[t] = 0.0f;
+        for (int c = c0 + lane; c < c1; c += 32) {
+            float uf[kEl], gf[kEl];
+            EL::unpack(reinterpret_cast<const uint4*>(us)[c], uf);
+            if (gated) EL::unpack(reinterpret_cast<const uint4*>(gs)[c], gf);
+#pragma unroll
+            for (int t = 0; t < TS; t++) {
+                if (t < T) {
+                    float xf[kEl];
+                    EL::unpack(reinterpret_cast<const uint4*>(xs + (size_t)t * d)[c], xf);
+#pragma unroll
+                    for (int q = 0; q < kEl; q++) au[t] = fmaf(uf[q], xf[q], au[t]);
+                    if (gated)
+#pragma unroll
+                        for (int q = 0; q < kEl; q++) ag[t] = fmaf(gf[q], xf[q], ag[t]);
+                }
+            }
+        }
+#pragma unroll
+        for (int t = 0; t < TS; t++) {
+            au[t] = warp_sum(au[t]);
+            ag[t] = gated ? warp_sum(ag[t]) : 0.0f;
+        }
+    };
+    auto store_h = [&](int i, int t, float su, float sg) {
+        const int q = nb + i;
+        const int u = q >> 6, n = q & 63;
+        const float w = gw[t * E + ulist[u]];
+        a.h_ws[((size_t)u * T + t) * kDExpert + n] = w == 0.0f ? 0.0f : act_h(a.act, su, sg) * w;
+    };
+    // Few neurons (cnt <= NS4): all loads at once, neuron i -> slot i, each
+    // neuron split into S column slices worked on by S warps.  Many neurons:
+    // warp w streams neurons w, w + NS4, ... through slot w.  The phase-4
+    // loads go into the copy queue before the phase-6 prefetch.
+    const bool few = cnt > 0 && cnt <= a.NS4;
+    if (few && tid == 0) {
+        fence_proxy_async_smem();
+        for (int i = 0; i < cnt; i++) issue4(i, i);
+    }
+    if (!few && warp < a.NS4 && cnt > warp && lane == 0) {
+        fence_proxy_async_smem();
+        issue4(warp, warp);
+    }
+    __syncwarp();
     if (lane == 0) {
         fence_proxy_async_smem();
-        if (ph4) issue4(warp);
         for (int i = 0; i < min(nt_w, ded6); i++) issue6(i);  // phase-6 prefetch
     }
-    if (ph4) {
-        uint32_t use = 0;
-        const TW* gs = reinterpret_cast<const TW*>(slot4);
-        const TW* us = reinterpret_cast<const TW*>(gated ? slot4 + rowb : slot4);
-        for (int i = warp; i < cnt; i += a.NS4) {
-            mbar_wait(fb4, use & 1u, a.status, lim);
-            use++;
+    if (few) {
+        const int S = cnt == 1 ? 8 : cnt == 2 ? 4 : cnt <= 4 ? 2 : 1;
+        if (warp < cnt * S) {
+            const int i = warp / S, sl = warp % S;
+            const int cs = (nchunk + S - 1) / S;
+            mbar_wait(&bars[kBarFull4 + i], 0, a.status, lim);
             float au[TS], ag[TS];
+            neuron_dots(i, sl * cs, min(nchunk, (sl + 1) * cs), au, ag);
 #pragma unroll
-            for (int t = 0; t < TS; t++) au[t] = ag[t] = 0.0f;
-            for (int c = lane; c < nchunk; c += 32) {
-                float uf[kEl], gf[kEl];
-                EL::unpack(reinterpret_cast<const uint4*>(us)[c], uf);
-                if (gated) EL::unpack(reinterpret_cast<const uint4*>(gs)[c], gf);
-#pragma unroll
-                for (int t = 0; t < TS; t++) {
-                    if (t < T) {
-                        float xf[kEl];
-                        EL::unpack(reinterpret_cast<const uint4*>(xs + (size_t)t * d)[c], xf);
-#pragma unroll
-                        for (int q = 0; q < kEl; q++) au[t] = fmaf(uf[q], xf[q], au[t]);
-                        if (gated)
-#pragma unroll
-                            for (int q = 0; q < kEl; q++) ag[t] = fmaf(gf[q], xf[q], ag[t]);
+            for (int t = 0; t < TS; t++) {
+                if (lane == t && t < T) {
+                    if (S == 1) {
+                        store_h(i, t, au[t], ag[t]);
+                    } else {
+                        red[(warp * 2 + 0) * TS + t] = au[t];
+                        red[(warp * 2 + 1) * TS + t] = ag[t];
                     }
                 }
             }
-            const int q = nb + i;
-            const int u = q >> 6, n = q & 63;
-            const int e = ulist[u];
-#pragma unroll
-            for (int t = 0; t < TS; t++) {
-                const float su = warp_sum(au[t]);
-                const float sg = gated ? warp_sum(ag[t]) : 0.0f;
-                if (lane == t && t < T) {
-                    const float w = gw[t * E + e];
-                    a.h_ws[((size_t)u * T + t) * kDExpert + n] = w == 0.0f ? 0.0f : act_h(a.act, su, sg) * w;
+        }
+        if (S > 1) {
+            __syncthreads();
+            if (tid < cnt * T) {
+                const int i = tid / T, t = tid % T;
+                float su = 0.0f, sg = 0.0f;
+                for (int sl = 0; sl < S; sl++) {
+                    su += red[((i * S + sl) * 2 + 0) * TS + t];
+                    sg += red[((i * S + sl) * 2 + 1) * TS + t];
                 }
+                store_h(i, t, su, sg);
             }
+        }
+    } else if (cnt > 0 && warp < a.NS4 && cnt > warp) {
+        uint32_t use = 0;
+        for (int i = warp; i < cnt; i += a.NS4) {
+            mbar_wait(&bars[kBarFull4 + warp], use & 1u, a.status, lim);
+            use++;
+            float au[TS], ag[TS];
+            neuron_dots(warp, 0, nchunk, au, ag);
+#pragma unroll
+            for (int t = 0; t < TS; t++)
+                if (lane == t && t < T) store_h(i, t, au[t], ag[t]);
             __syncwarp();
             if (lane == 0 && i + a.NS4 < cnt) {
                 fence_proxy_async_smem();
-                issue4(i + a.NS4);
+                issue4(i + a.NS4, warp);
             }
         }
     }
@@ -494,12 +552,20 @@ static cudaError_t launch_one(const DecodeArgs& a, const DecodePlan& p, int grid
     cfg.blockDim = dim3(p.threads);
     cfg.dynamicSmemBytes = p.smem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeCooperative;
     attr[0].val.cooperative = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, a);
+    cfg.numAttrs = 2;
+    e = cudaLaunchKernelEx(&cfg, kern, a);
+    if (e == cudaErrorNotSupported || e == cudaErrorInvalidValue) {
+        (void)cudaGetLastError();  // this runtime cannot combine the two attributes
+        cfg.numAttrs = 1;
+        e = cudaLaunchKernelEx(&cfg, kern, a);
+    }
+    return e;
 }
 
 template <typename TW, int TS>

@@ -112,6 +112,12 @@ PP_DEVINL void tma_load_2d(void* dst, const CUtensorMap* map, int c0, int c1, ui
         : "memory");
 }
 
+// Programmatic dependent launch: wait until the preceding grid on the stream
+// has completed and its memory is visible (no-op when launched without the
+// attribute); allow the next grid on the stream to start launching.
+PP_DEVINL void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+PP_DEVINL void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // Order this thread's earlier generic-proxy shared-memory accesses before
 // later async-proxy (TMA) accesses of the same memory.
 PP_DEVINL void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }

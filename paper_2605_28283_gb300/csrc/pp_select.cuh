@@ -153,12 +153,12 @@ PP_DEVINL float gate_of(int gate_mode, unsigned long long k) {
 // e_j = exp(g_j - max g) (fp32) are summed as exact 2^-31 fixed-point
 // integers, and the cut compares S against p * Z exactly in integers, so
 // the only rounding is that of the fp32 exponentials.
-//   MIN_PREFIX: j selected  <=>  r_j == 0  or  S_{r_j - 1} <  p Z
-//   PAPER:      j selected  <=>  r_j == 0  or  S_{r_j}     <  p Z
+//   MIN_PREFIX: j activated <=> r_j == 0  or  S_{r_j - 1} <  p Z
+//   PAPER:      j activated <=> r_j == 0  or  S_{r_j}     <  p Z
 // (S non-decreasing along the order, so both are prefixes of the order.)
 
 struct CtaSelScratch {
-    uint32_t D[kMaxExperts];  // descending-order keys (ascending = larger logit)
+    uint32_t D[kMaxExperts];  // descending-order keys (smaller = larger logit)
     uint32_t U[kMaxExperts];  // fixed-point exponentials, e * 2^31
     float fred[8];
     unsigned long long ured[8];
@@ -186,31 +186,34 @@ PP_DEVINL long long prefix_threshold(float p, unsigned long long Z) {
 }
 
 // Returns the activated count (CTA-uniform).  On return: *sel = whether
-// expert j (= threadIdx.x) is activated, *rank = its rank (valid j only),
-// *gval = its logit.  All threads of the CTA must call it.
+// expert j (= threadIdx.x) is activated, *rank = its rank, *gval = its
+// logit.  All threads of the CTA (8 warps) must call it.
 template <typename Load>
 PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, CtaSelScratch& sc, unsigned* status,
                             bool* sel, int* rank, float* gval) {
     const int j = threadIdx.x;
-    const int lane = j & 31, warp = j >> 5, nwarps = blockDim.x >> 5;
+    const int lane = j & 31, warp = j >> 5;
     const bool valid = j < E;
     const float g = valid ? load(j) : -INFINITY;
     *gval = g;
+    *rank = j;
     const bool fin = !valid || isfinite(g);
     if (!__syncthreads_and(fin)) {
         if (j == 0) record_status(status, PP_ERR_NONFINITE);
         *sel = false;
-        *rank = j;
         return 0;
     }
-    // max logit
+    // max logit: warp shuffles, then the 8 warp maxima read as two vectors
     float m = g;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(kFull, m, o));
     if (lane == 0) sc.fred[warp] = m;
     __syncthreads();
-    m = sc.fred[0];
-    for (int w = 1; w < nwarps; w++) m = fmaxf(m, sc.fred[w]);
+    {
+        const float4 a = *reinterpret_cast<const float4*>(&sc.fred[0]);
+        const float4 b = *reinterpret_cast<const float4*>(&sc.fred[4]);
+        m = fmaxf(fmaxf(fmaxf(a.x, a.y), fmaxf(a.z, a.w)), fmaxf(fmaxf(b.x, b.y), fmaxf(b.z, b.w)));
+    }
     // fixed-point exponentials and their sum Z
     const float e = valid ? expf(g - m) : 0.0f;
     const uint32_t U = valid ? __float2uint_rn(e * 2147483648.0f) : 0u;
@@ -222,33 +225,33 @@ PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, CtaSelScratch& 
     for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(kFull, z, o);
     if (lane == 0) sc.ured[warp] = z;
     __syncthreads();
-    unsigned long long Z = 0;
-    for (int w = 0; w < nwarps; w++) Z += sc.ured[w];
-    // rank and exclusive prefix mass by counting the experts ahead: first the
-    // strictly larger logits, then (rare) equal logits with a lower index --
-    // equal logits have equal exponentials, so they add U once each
-    int r = 0, eq = 0;
-    unsigned long long ahead_mass = 0;
+    unsigned long long Z;
+    {
+        const ulonglong2* v = reinterpret_cast<const ulonglong2*>(sc.ured);
+        const ulonglong2 a = v[0], b = v[1], c = v[2], d2 = v[3];
+        Z = (a.x + a.y) + (b.x + b.y) + (c.x + c.y) + (d2.x + d2.y);
+    }
+    // rank and exclusive prefix mass: experts with a strictly larger logit,
+    // four independent accumulator chains; equal logits are counted too and
+    // resolved by index afterwards (rare; equal logits have equal U)
+    int r0 = 0, r1 = 0, r2 = 0, r3 = 0, eq = 0;
+    unsigned long long m0 = 0, m1 = 0, m2 = 0, m3 = 0;
     const int E4 = E & ~3;
     for (int i = 0; i < E4; i += 4) {
         const uint4 d4 = *reinterpret_cast<const uint4*>(&sc.D[i]);
         const uint4 u4 = *reinterpret_cast<const uint4*>(&sc.U[i]);
-        const uint32_t dd[4] = {d4.x, d4.y, d4.z, d4.w};
-        const uint32_t uu[4] = {u4.x, u4.y, u4.z, u4.w};
-#pragma unroll
-        for (int q = 0; q < 4; q++) {
-            const bool lt = dd[q] < D;
-            r += lt ? 1 : 0;
-            eq += dd[q] == D ? 1 : 0;
-            ahead_mass += lt ? (unsigned long long)uu[q] : 0ull;
-        }
+        r0 += d4.x < D; m0 += d4.x < D ? (unsigned long long)u4.x : 0ull; eq += d4.x == D;
+        r1 += d4.y < D; m1 += d4.y < D ? (unsigned long long)u4.y : 0ull; eq += d4.y == D;
+        r2 += d4.z < D; m2 += d4.z < D ? (unsigned long long)u4.z : 0ull; eq += d4.z == D;
+        r3 += d4.w < D; m3 += d4.w < D ? (unsigned long long)u4.w : 0ull; eq += d4.w == D;
     }
     for (int i = E4; i < E; i++) {
-        const bool lt = sc.D[i] < D;
-        r += lt ? 1 : 0;
-        eq += sc.D[i] == D ? 1 : 0;
-        ahead_mass += lt ? (unsigned long long)sc.U[i] : 0ull;
+        r0 += sc.D[i] < D;
+        m0 += sc.D[i] < D ? (unsigned long long)sc.U[i] : 0ull;
+        eq += sc.D[i] == D;
     }
+    int r = (r0 + r1) + (r2 + r3);
+    unsigned long long ahead_mass = (m0 + m1) + (m2 + m3);
     if (valid && eq > 1) {  // ties: the equal logits of lower index are ahead
         int tb = 0;
         for (int i = 0; i < j; i++) tb += sc.D[i] == D ? 1 : 0;
@@ -265,8 +268,7 @@ PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, CtaSelScratch& 
     }
     *sel = on;
     *rank = r;
-    const int k = __syncthreads_count(on);
-    return k;
+    return __syncthreads_count(on);
 }
 
 // Same, reading the logits (written by other CTAs earlier) from a row.
@@ -274,5 +276,6 @@ PP_DEVINL int cta_select(const float* __restrict__ logits_row, int E, float p, i
                          unsigned* status, bool* sel, int* rank, float* gval) {
     return cta_select_fn([&](int j) { return __ldcg(logits_row + j); }, E, p, rule, sc, status, sel, rank, gval);
 }
+
 
 }  // namespace pp

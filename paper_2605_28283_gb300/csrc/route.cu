@@ -33,18 +33,18 @@ __global__ void __launch_bounds__(256) select_kernel(const float* __restrict__ l
 }
 
 // One CTA per token (the latency-oriented counting selection of
-// pp_select.cuh); used for small token counts.
-__global__ void __launch_bounds__(256) select_cta_kernel(const float* __restrict__ logits, int E, float p,
-                                                         int rule, int gate, int32_t* ids, int32_t* counts,
-                                                         float* gates, unsigned* status) {
+// pp_select.cuh, the one the fused decode kernel runs); used for small T.
+__global__ void __launch_bounds__(256) select_cta_kernel(const float* __restrict__ logits, int E, float p, int rule,
+                                                         int gate, int32_t* ids, int32_t* counts, float* gates,
+                                                         unsigned* status) {
     __shared__ __align__(16) CtaSelScratch sc;
     const int t = blockIdx.x;
     bool on;
     int r;
     float g;
-    const int k = cta_select(logits + (size_t)t * E, E, p, rule, sc, status, &on, &r, &g);
+    const int k = cta_select_fn([&](int j) { return logits[(size_t)t * E + j]; }, E, p, rule, sc, status, &on, &r, &g);
     const int j = threadIdx.x;
-    if (j < E) {
+    if (j < E) {  // ranks are a permutation: every rank slot is written once
         ids[(size_t)t * E + r] = on ? j : -1;
         gates[(size_t)t * E + r] = on ? (gate == PP_GATE_NONE ? 1.0f : sigmoidf_(g)) : 0.0f;
     }
