@@ -40,7 +40,8 @@ def parse():
     ap.add_argument("--workload", default="llama2_7b_decode")
     ap.add_argument("--p", type=float, default=0.7)
     ap.add_argument("--batch", type=int, default=1)
-    ap.add_argument("--pool", type=int, default=16, help="distinct token vectors per layer")
+    ap.add_argument("--pool", type=int, default=0,
+                    help="distinct token sets per layer (default 16 for decode batches, 1 for prefill)")
     ap.add_argument("--sweep", default="0.3,0.5,0.7,0.9,1.0", help="p values for the sweep ('' = none)")
     ap.add_argument("--sweep-steps", type=int, default=400)
     ap.add_argument("--no-flush", action="store_true")
@@ -60,12 +61,14 @@ def dist_env():
 
 
 def load_peaks():
+    """(HBM GB/s, dense bf16 TFLOP/s sustained, kind): measured copy and GEMM
+    figures for this GPU pool, else the recipe's fallback numbers."""
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
             pk = json.load(f)
-        return float(pk["hbm_gbs"]), "measured"
+        return float(pk["hbm_gbs"]), float(pk.get("bf16_tflops_sustained", pk["bf16_tflops"])), "measured"
     except Exception:
-        return 6800.0, "fallback"
+        return 6800.0, 1700.0, "fallback"
 
 
 # --------------------------------------------------------------- clocks
@@ -149,8 +152,10 @@ def capture_graphs(pp, desc, layers, p, B, pool, ws, stream):
     return graphs
 
 
-def time_graphs(graphs, steps, warmup, flush_buf, stream):
-    """Per-step CUDA-event timing on `stream`; L2 flushed between steps."""
+def time_graphs(graphs, steps, warmup, flush_buf, stream, profile_range=False):
+    """Per-step CUDA-event timing on `stream`; L2 flushed between steps.
+    With profile_range, the timed loop is bracketed by cudaProfilerStart/Stop
+    so that `ncu --profile-from-start off` lists exactly its launches."""
     import torch
     with torch.cuda.stream(stream):
         for i in range(warmup):
@@ -158,6 +163,8 @@ def time_graphs(graphs, steps, warmup, flush_buf, stream):
         stream.synchronize()
         ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
               for _ in range(steps)]
+        if profile_range:
+            torch.cuda.profiler.start()
         for i in range(steps):
             if flush_buf is not None:
                 flush_buf.add_(1)
@@ -165,11 +172,14 @@ def time_graphs(graphs, steps, warmup, flush_buf, stream):
             graphs[i % len(graphs)].replay()
             ev[i][1].record(stream)
         stream.synchronize()
+        if profile_range:
+            torch.cuda.profiler.stop()
     return [a.elapsed_time(b) for a, b in ev]  # ms
 
 
 def selection_stats(pp, desc, layers, w, p, B, pool, ws):
     """k per (pool entry, layer, token) via pp_route on the same inputs."""
+    import numpy as np
     import torch
     ks = torch.empty((pool, len(layers), B), dtype=torch.int64)
     union = torch.empty((pool, len(layers)), dtype=torch.int64)
@@ -179,16 +189,15 @@ def selection_stats(pp, desc, layers, w, p, B, pool, ws):
             pp.pp_route(desc, L["x"][i], B, L["Wr"], p, sel, ws)
             c = sel.counts.cpu()
             ks[i, l] = c.long()
-            ids = sel.ids.cpu()
-            u = set()
-            for t in range(B):
-                u.update(ids[t, :int(c[t])].tolist())
-            union[i, l] = len(u)
+            ids = sel.ids.cpu().numpy()
+            cn = c.numpy()
+            mask = np.arange(ids.shape[1])[None, :] < cn[:, None]
+            union[i, l] = len(np.unique(ids[mask]))
     return ks, union
 
 
 def layer_bytes(w, B, n_union):
-    """Algorithmic HBM bytes of one pp_layer launch: W_r, the union of the
+    """Algorithmic HBM bytes of one pp_layer call: W_r, the union of the
     selected expert blocks (gate+up rows and down column block), x and y."""
     esz = 2 if w.dtype == "bf16" else 4
     mats = 3 if w.gated else 2
@@ -198,18 +207,25 @@ def layer_bytes(w, B, n_union):
     return router + n_union * expert + act, n_union * expert
 
 
-def kernel_traffic(workload, p):
-    """DRAM bytes per launch of the layer kernel from a committed ncu summary,
-    valid only while the kernel sources are unchanged."""
-    path = os.path.join(ROOT, "profiles", "decode_layer_traffic.json")
+def layer_flops(w, B, k_sum):
+    """Algorithmic FLOPs of one pp_layer call: router GEMV/GEMM plus, per
+    (token, activated expert), the gate/up and down products of a 64-wide block."""
+    mats = 3 if w.gated else 2
+    return 2.0 * B * w.n_experts * w.d_model + 2.0 * k_sum * mats * 64 * w.d_model
+
+
+def kernel_traffic(workload, p, B):
+    """DRAM bytes per layer call measured by ncu (committed summary), valid
+    only while the kernel sources are unchanged; None otherwise."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic.json")
     try:
         rec = json.load(open(path))
     except Exception:
         return None
     if rec.get("sources_sha") != sources_sha():
         return None
-    ent = rec.get("entries", {}).get("%s@%g" % (workload, p))
-    return None if ent is None else ent.get("dram_bytes_per_launch")
+    ent = rec.get("entries", {}).get("%s@p%g@B%d" % (workload, p, B))
+    return None if ent is None else ent.get("dram_bytes_per_layer")
 
 
 def sources_sha():
@@ -290,6 +306,8 @@ def run_reference(args):
 # ------------------------------------------------------------------ main
 def main():
     args = parse()
+    if args.pool <= 0:
+        args.pool = 16 if args.batch <= 128 else 1
     if args.impl == "reference":
         return run_reference(args)
     import numpy as np
@@ -335,7 +353,7 @@ def main():
     sampler = ClockSampler(local)
     barrier()
     sampler.start()
-    times = time_graphs(graphs, args.steps, args.warmup, flush, stream)
+    times = time_graphs(graphs, args.steps, args.warmup, flush, stream, profile_range=True)
     barrier()
     clocks = sampler.stop()
     total_ms = max_over_ranks(sum(times))
@@ -348,19 +366,33 @@ def main():
     # bytes per step from the actual selections of the pool entries
     ks, union = selection_stats(pp, desc, layers, w, pf, B, args.pool, ws)
     step_ids = np.arange(args.steps) % args.pool
-    tot_b, exp_b = 0.0, 0.0
+    tot_b, exp_b, tot_f = 0.0, 0.0, 0.0
     for i in range(args.pool):
         n_i = int((step_ids == i).sum())
         for l in range(w.n_layers):
             a, e = layer_bytes(w, B, int(union[i, l]))
             tot_b += n_i * a
             exp_b += n_i * e
+            tot_f += n_i * layer_flops(w, B, int(ks[i, l].sum()))
     seconds = sum(times) / 1e3
     launches = args.steps * w.n_layers
+    # kernels of ours per layer call: the fused decode kernel (<= 4 bf16 / 8 fp32
+    # tokens), else router, selection, 4 dispatch kernels, gate/up, down, combine
+    kernels_per_layer = 1 if (B <= 4 or w.dtype == "f32") else 9
     per_launch_ms = sum(times) / launches   # step time / L: includes the in-graph launch gaps
     bytes_per_launch = tot_b / launches
-    peak, peak_kind = load_peaks()
-    achieved = bytes_per_launch / (per_launch_ms / 1e3) / 1e9
+    flops_per_launch = tot_f / launches
+    hbm_peak, tc_peak, peak_kind = load_peaks()
+    # the bound is whichever of HBM traffic and tensor work takes longer at peak
+    tensor_bound = flops_per_launch / (tc_peak * 1e12) > bytes_per_launch / (hbm_peak * 1e9)
+    if tensor_bound:
+        achieved = flops_per_launch / (per_launch_ms / 1e3) / 1e12
+        peak = tc_peak
+        roof = {"bound": "tensor", "unit": "TFLOP/s", "flops_per_launch": flops_per_launch}
+    else:
+        achieved = bytes_per_launch / (per_launch_ms / 1e3) / 1e9
+        peak = hbm_peak
+        roof = {"bound": "hbm", "unit": "GB/s", "bytes_per_launch": bytes_per_launch}
     expert_gbs = exp_b / seconds / 1e9
     k_mean = float(ks.float().mean())
     s_ffn = 1.0 - k_mean / w.n_experts
@@ -382,7 +414,7 @@ def main():
             sweep["%g" % ps] = {"tokens_per_s": B * args.sweep_steps / sec, "ms_per_step": sum(tm) / args.sweep_steps,
                                 "k_mean": float(kk.float().mean()), "s_ffn": 1 - float(kk.float().mean()) / w.n_experts,
                                 "expert_gbs": eb / sec / 1e9, "total_gbs": tb / sec / 1e9,
-                                "frac_of_peak_total": tb / sec / 1e9 / peak}
+                                "frac_of_hbm_peak": tb / sec / 1e9 / hbm_peak}
             del gs
         dense = sweep.get("1")
         if dense:
@@ -392,8 +424,11 @@ def main():
     if args.skip_extras:
         if rank == 0:
             print(json.dumps({"metric": METRIC, "value": value, "unit": "tokens/s", "ms_per_step": ms_per_step,
-                              "workload": w.name, "layers": w.n_layers, "p": args.p,
-                              "launch_ms": per_launch_ms, "bytes_per_launch": bytes_per_launch}))
+                              "workload": w.name, "layers": w.n_layers, "p": args.p, "batch": B,
+                              "launch_ms": per_launch_ms, "bytes_per_launch": bytes_per_launch,
+                              "flops_per_launch": flops_per_launch, "roofline_bound": roof["bound"],
+                              "achieved": achieved, "peak": peak, "frac": achieved / peak,
+                              "sources_sha": sources_sha()}))
         return
 
     # ---- warm-L2 number (no flush), for context
@@ -433,14 +468,15 @@ def main():
                       "token_pool": args.pool,
                       "l2": "no flush (warm)" if args.no_flush else "flushed between steps (256 MiB write, untimed)",
                       "parallelism": "replicas" if world > 1 else "single GPU"},
-           "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                        "frac": achieved / peak, "traffic": kernel_traffic(w.name, args.p),
-                        "peak_kind": peak_kind, "kernel": "decode_layer_kernel",
-                        "bytes_per_launch": bytes_per_launch, "launch_ms": per_launch_ms},
-           "expert_bytes": {"gbs": expert_gbs, "frac_of_peak": expert_gbs / peak,
+           "roofline": dict(roof, achieved=achieved, peak=peak, frac=achieved / peak,
+                            traffic=kernel_traffic(w.name, args.p, B), peak_kind=peak_kind,
+                            kernel="decode_layer_kernel" if B <= 4 else "pp_layer (grouped tcgen05 path)",
+                            per="one pp_layer call (one layer)", launch_ms=per_launch_ms),
+           "expert_bytes": {"gbs": expert_gbs, "frac_of_peak": expert_gbs / hbm_peak,
                             "frac_of_8tbs": expert_gbs / 8000.0, "k_mean": k_mean, "s_ffn": s_ffn},
+           "hbm_gbs_total": tot_b / seconds / 1e9, "tflops": tot_f / seconds / 1e12,
            "p_sweep": sweep, "warm_l2_tokens_per_s": warm_tok_s,
-           "e2e": e2e, "gpu_launches": launches, "clocks": clocks}
+           "e2e": e2e, "gpu_launches": launches * kernels_per_layer, "clocks": clocks}
     if rank == 0 and world == 1:
         try:
             out["cpu_baseline"] = run_oracle_sample(w, args.cpu_seconds, args.seed, p=args.p, B=B)

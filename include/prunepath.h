@@ -116,7 +116,9 @@ pp_status pp_workspace_init(void *ws, size_t ws_bytes, void *stream);
 /* Router and selection (Eq. routing_logits, softmax_prob,
    tau_thresh_activate).  x [T][d], W_r [E][d]; writes *out (out->logits may
    be NULL).  The softmax is max-shifted in fp32 with fp32 exponentials; the
-   normaliser and the prefix masses are accumulated in fp64; the order is
+   normaliser and the prefix masses are summed exactly (2^-31 fixed-point
+   integers for up to 64 tokens per call, fp64 beyond), so the cut is decided
+   by an exact comparison with p times the normaliser; the order is
    descending logit with ties broken by the lower expert index. */
 pp_status pp_route(const pp_desc *desc, const void *x, int T, const void *W_r, float p,
                    const pp_selection *out, void *ws, size_t ws_bytes, void *stream);
