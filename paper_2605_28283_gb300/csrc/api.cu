@@ -180,9 +180,12 @@ bool make_down_map(const pp_desc& d, const void* Wd, int R6, CUtensorMap* map) {
     const cuuint64_t strides[1] = {(cuuint64_t)d.d_ff * (bf ? 2 : 4)};
     const cuuint32_t box[2] = {(cuuint32_t)kDExpert, (cuuint32_t)R6};
     const cuuint32_t estr[2] = {1, 1};
+    // 128-byte L2 fills for bf16: the next 128 bytes of a row belong to the
+    // neighbouring expert, which is usually not selected
     const CUresult r = enc(map, bf ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2,
                            const_cast<void*>(Wd), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                           CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                           CU_TENSOR_MAP_SWIZZLE_NONE,
+                           bf ? CU_TENSOR_MAP_L2_PROMOTION_L2_128B : CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }

@@ -621,8 +621,12 @@ __global__ void __launch_bounds__(128) combine_kernel(const uint32_t* __restrict
 // ====================================================================== host
 namespace {
 
+// bf16 [outer][inner] row-major, SW128 boxes.  `promote` is the L2 fill
+// granularity: 256 B where the neighbouring 128 B of a row is read next by
+// the same CTA (K-major operand streams), 128 B where it belongs to another
+// expert that may not be selected (the 64-column blocks of W_down).
 bool encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer, uint32_t box_inner,
-               uint32_t box_outer) {
+               uint32_t box_outer, CUtensorMapL2promotion promote = CU_TENSOR_MAP_L2_PROMOTION_L2_256B) {
     auto enc = tensor_map_encoder();
     if (!enc) return false;
     const cuuint64_t dims[2] = {inner, outer};
@@ -630,7 +634,7 @@ bool encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t oute
     const cuuint32_t box[2] = {box_inner, box_outer};
     const cuuint32_t estr[2] = {1, 1};
     return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, promote,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -719,7 +723,7 @@ cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
     if (!encode_2d(&mx1, a.x, a.d, a.T, 64, 1) || !encode_2d(&mwu, a.Wu, a.d, (uint64_t)a.E * 64, 64, 64) ||
         !encode_2d(&mwg, gated ? a.Wg : a.Wu, a.d, (uint64_t)a.E * 64, 64, 64) ||
         !encode_2d(&mh, a.H, 64, (uint64_t)g.nnz_max + 128, 64, 128) ||
-        !encode_2d(&mwd, a.Wd, (uint64_t)a.E * 64, a.d, 64, 256))
+        !encode_2d(&mwd, a.Wd, (uint64_t)a.E * 64, a.d, 64, 256, CU_TENSOR_MAP_L2_PROMOTION_L2_128B))
         return cudaErrorInvalidValue;
     const int grid = std::max(1, std::min(sms, g.max_items));
     const WorkItem* items = reinterpret_cast<const WorkItem*>(a.items);
