@@ -36,7 +36,8 @@
  *  - Workspace: caller-owned device memory of at least pp_workspace_size()
  *    bytes, 256-byte aligned, zeroed once by pp_workspace_init before its
  *    first use.  Calls that share a workspace must be ordered on one stream;
- *    calls on different workspaces are independent.
+ *    calls on different workspaces are independent.  A workspace serves one
+ *    device (it keeps per-SM launch counts of the fused decode kernel).
  *  - No C++ exception crosses this interface.
  *  - Supported shapes: d_expert == 64, d_ff == E * 64, 1 <= E <= 256,
  *    d a multiple of 8 (bf16) or 4 (fp32), 64 <= d <= 8192, T >= 0.
@@ -108,7 +109,7 @@ typedef struct pp_selection {
 /* Bytes of workspace needed for calls with up to T tokens. */
 size_t pp_workspace_size(const pp_desc *desc, int T);
 
-/* Zero the whole workspace (status word, barrier counters, accumulators) on
+/* Zero the whole workspace (status word, launch counts, accumulators) on
    `stream`.  Call once after allocating a workspace, and again to clear a
    sticky device error. */
 pp_status pp_workspace_init(void *ws, size_t ws_bytes, void *stream);
@@ -147,15 +148,16 @@ pp_status pp_layer(const pp_desc *desc, const void *x, int T, const void *W_r, c
    that exposes no allocator.  The paper has no counterpart: this entry point
    exists only for those callers.
    Same computation and arguments as pp_layer, for T <= 4 tokens and without a
-   workspace.  Its scratch (status word, barrier counter, router logits, gate/up
-   activations: 266,496 bytes) is one static device array that every GPU loading
-   this library keeps until the process exits; no call allocates or frees.
+   workspace.  Its scratch (status word, per-CTA launch counts, router
+   logits and gate/up activations: 533,760 bytes) is one static
+   device array that every GPU loading this library keeps until the process
+   exits; no call allocates or frees.
    - T > 4 (like any shape pp_layer rejects) returns PP_ERR_SHAPE.
    - The first call on a device, made with that device current, looks up the
      array's address there; make that first call before any stream capture.
-   - Every call reuses the same array and first clears its status word and
-     barrier counter; calls that overlap on the GPU (other streams, other host
-     threads) race on it, so the caller must serialise them.
+   - Every call reuses the same array and first clears its status word;
+     calls that overlap on the GPU (other streams, other host threads) race
+     on it, so the caller must serialise them.
    - status_out (optional, device uint32) receives the call's device-side
      status (a pp_status code) when the call has run on `stream`. */
 pp_status pp_layer_noalloc(const pp_desc *desc, const void *x, int T, const void *W_r,

@@ -52,7 +52,7 @@ bool use_grouped(const pp_desc& d, int T) { return d.dtype == PP_BF16 && T >= kG
 
 // Workspace layout for calls with up to T tokens.
 struct Layout {
-    size_t logits, ids, counts, gates, h;
+    size_t logits, ids, counts, gates, tlog, th;
     // grouped path
     size_t part, bits, gexp, invpos, wcnt, blkcnt, blkbase, offsets, n_items, items, perm_token, perm_gate, H, Y,
         yacc, overflow;
@@ -72,7 +72,9 @@ Layout layout(const pp_desc& d, int T) {
     L.ids = take(Tn * E * 4);
     L.counts = take(Tn * 4);
     L.gates = take(Tn * E * 4);
-    L.h = take(E * 8 * kDExpert * 4);
+    // tagged exchange words of the fused decode kernel (up to 8 tokens a launch)
+    L.tlog = take(8 * E * 8);
+    L.th = take(E * 8 * kDExpert * 8);
     if (use_grouped(d, T)) {
         const GroupedPlan g = grouped_plan(T, d.d_model, d.n_experts, 152);
         L.part = take((size_t)g.nsplit * Tn * E * 4);
@@ -161,7 +163,8 @@ struct Ws {
     int32_t* ids;
     int32_t* counts;
     float* gates;
-    float* h;
+    unsigned long long* tlog;
+    unsigned long long* th;
 };
 
 Ws ws_views(const pp_desc& d, int T, void* ws) {
@@ -169,7 +172,8 @@ Ws ws_views(const pp_desc& d, int T, void* ws) {
     char* b = static_cast<char*>(ws);
     return Ws{reinterpret_cast<Control*>(b), reinterpret_cast<float*>(b + L.logits),
               reinterpret_cast<int32_t*>(b + L.ids), reinterpret_cast<int32_t*>(b + L.counts),
-              reinterpret_cast<float*>(b + L.gates), reinterpret_cast<float*>(b + L.h)};
+              reinterpret_cast<float*>(b + L.gates), reinterpret_cast<unsigned long long*>(b + L.tlog),
+              reinterpret_cast<unsigned long long*>(b + L.th)};
 }
 
 bool make_down_map(const pp_desc& d, const void* Wd, int R6, CUtensorMap* map) {
@@ -192,9 +196,8 @@ bool make_down_map(const pp_desc& d, const void* Wd, int R6, CUtensorMap* map) {
 
 DecodePlanIn plan_in(const pp_desc& d, int TS) {
     const DeviceInfo di = device_info();
-    // leave 4 KB of the opt-in limit for the kernel's static shared memory
-    // (selection scratch and counters, under 3 KB)
-    return DecodePlanIn{d.dtype, d.d_model, d.n_experts, TS, di.sms, d.act == PP_ACT_SWIGLU, di.smem_optin - 4096};
+    return DecodePlanIn{d.dtype, d.d_model, d.n_experts, TS, di.sms, d.act == PP_ACT_SWIGLU,
+                        di.smem_optin - kDecodeStaticSmemReserve};
 }
 
 // Largest token count one fused decode launch takes for this shape (0: none).
@@ -276,10 +279,10 @@ pp_status decode_call(const pp_desc& d, const void* x, int t0, int n, const void
         a.sel_gates = sel->gates + (size_t)t0 * E;
         a.sel_logits = sel->logits ? sel->logits + (size_t)t0 * E : nullptr;
     }
-    a.logit_ws = w.logits;
-    a.h_ws = w.h;
+    a.tlog = w.tlog;
+    a.th = w.th;
+    a.epochs = w.ctrl->epoch;
     a.status = &w.ctrl->status;
-    a.bar = &w.ctrl->grid_bar[0];
     a.timeout_ns = kDefaultTimeoutNs;
     a.T = n;
     a.d = d.d_model;
@@ -294,7 +297,7 @@ pp_status decode_call(const pp_desc& d, const void* x, int t0, int n, const void
     a.NS4 = plan.NS4;
     a.ded6 = plan.ded6;
     a.slots6 = plan.slots6;
-    a.uch = plan.uch;
+    a.hch = plan.hch;
     a.off_x = plan.off_x;
     a.off_gw = plan.off_gw;
     a.off_mask = plan.off_mask;

@@ -3,26 +3,30 @@
 // One cooperative, persistent launch of one CTA (8 warps) per SM does, for
 // T <= TS tokens:
 //   phase 1  router (Eq. routing_logits): CTA b bulk-loads its rows of W_r
-//            and dots them with x (fp32 FMA), writing logits to the workspace;
-//   -- grid barrier --
-//   select   every CTA redundantly selects each token's experts with the
-//            CTA-parallel counting selection (Eq. softmax_prob, the
-//            descending order, Eq. tau_thresh_activate) and forms U, the
-//            union of the tokens' activated experts;
+//            and dots them with x (fp32 FMA), publishing each logit as a
+//            tagged word (pp_common.cuh);
+//   select   every CTA waits for the logits as they arrive, then redundantly
+//            selects each token's experts with the CTA-parallel counting
+//            selection (Eq. softmax_prob, the descending order, Eq.
+//            tau_thresh_activate) and forms U, the union of the tokens'
+//            activated experts;
 //   phase 4  gate/up (Eq. ffn on the expert blocks): the |U|*64 neurons are
 //            split evenly over the grid; each warp bulk-loads the gate and up
 //            rows of one neuron into its own shared-memory slot, computes
-//            h = act(.) * gate weight (Eq. moe_output) per token and stores
-//            it to the workspace;
-//   -- grid barrier --
+//            h = act(.) * gate weight (Eq. moe_output) per token and
+//            publishes it as a tagged word;
 //   phase 6  down projection: CTA b owns R6 rows of W_down and y.  Warp w
 //            handles the experts u = w, w+8, ... of U: it streams the
 //            [R6 x 64] column block of each with 2-D tensor TMA into its own
 //            slots (the first ones are issued before phase 4, so they
-//            overlap it) and accumulates every row of the CTA in registers;
-//            one cross-warp reduction in shared memory then writes y once
-//            (no atomics: deterministic).
-// Only the selected expert blocks are read from HBM.
+//            overlap it), waits for those experts' h words and accumulates
+//            every row of the CTA in registers; one cross-warp reduction in
+//            shared memory then writes y once (no atomics: deterministic).
+// There is no grid barrier: a CTA waits only for the words it reads.  Each
+// launch tags its words with the launch count of the CTA
+// (Control.epoch[b], the same in every CTA because every launch runs one CTA
+// per SM and each CTA adds 1 to its own count), so words of an earlier
+// launch never match.  Only the selected expert blocks are read from HBM.
 #include "pp_common.cuh"
 #include "pp_kernels.h"
 #include "pp_select.cuh"
@@ -35,8 +39,8 @@ constexpr int kMaxNS4 = kWarps;
 constexpr int kMaxSlots6 = 4;  // phase-6 slots per warp
 
 // barrier indices in the first bytes of shared memory
-constexpr int kBarX = 0, kBarR = 1, kBarH = 2, kBarFull4 = 3, kBarFull6 = kBarFull4 + kMaxNS4,
-              kNumBars = kBarFull6 + kWarps * kMaxSlots6;
+constexpr int kBarX = 0, kBarR = 1, kBarFull4 = 2, kBarFull6 = kBarFull4 + kMaxNS4,
+              kBarH = kBarFull6 + kWarps * kMaxSlots6, kNumBars = kBarH + kWarps;
 
 // Selection given by the caller (pp_sparse_ffn): gates are summed per expert
 // so repeated ids behave like repeated terms of the sum.
@@ -85,6 +89,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     __shared__ __align__(16) CtaSelScratch sel_sc;
     __shared__ int s_nU;
     __shared__ int s_wcount[kWarps];
+    __shared__ unsigned s_tag;
 
     if (tid == 0) {
         for (int i = 0; i < kNumBars; i++) mbar_init(&bars[i], 1);
@@ -111,14 +116,21 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     }
     pdl_wait();
     pdl_launch_dependents();
-    if (tid == 0) {  // x -> shared memory (all T rows are contiguous)
-        const uint32_t bytes = (uint32_t)(T * rowb);
+    if (tid == 0) {
+        const uint32_t bytes = (uint32_t)(T * rowb);  // x -> shared memory (all T rows are contiguous)
         mbar_arrive_expect_tx(&bars[kBarX], bytes);
         bulk_g2s(xs, a.x, bytes, &bars[kBarX]);
+        // this launch's tag: the CTA's launch count + 1 (its own word, last
+        // written by this CTA in the previous launch, which has completed)
+        const unsigned ep = a.epochs[b];
+        a.epochs[b] = ep + 1u;
+        s_tag = ep + 1u;
     }
     // every CTA waits for its copy of x here, so no bulk copy is ever still
     // in flight when a CTA that has no work left exits
     mbar_wait(&bars[kBarX], 0, a.status, lim);
+    __syncthreads();
+    const unsigned tag = s_tag;
 
     // ---------------------------------------------------------- phase 1
     if (a.do_route) {
@@ -161,20 +173,23 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
                     if (r0 + i < nrows && t < T) {
                         float v = 0.0f;
                         for (int w = 0; w < kWarps; w++) v += red[(w * 2 + i) * TS + t];
-                        a.logit_ws[(size_t)t * E + j0 + r0 + i] = v;
+                        st_tagged(a.tlog + (size_t)t * E + j0 + r0 + i, tag, v);
                     }
                 }
                 __syncthreads();
             }
         }
-        grid_barrier(a.bar, a.status, lim);
-        // selection of every token by the whole CTA; CTA 0 publishes it
+        // selection of every token by the whole CTA, from the tagged logits
+        // as they arrive; CTA 0 publishes it
         const bool publish = b == 0;
+        const bool want_rank = publish && a.sel_ids != nullptr;
         for (int t = 0; t < T; t++) {
             bool on;
             int r;
             float g;
-            const int k = cta_select(a.logit_ws + (size_t)t * E, E, a.p, a.rule, sel_sc, a.status, &on, &r, &g);
+            const unsigned long long* row = a.tlog + (size_t)t * E;
+            const int k = cta_select_fn([&](int j) { return wait_tagged(row + j, tag, a.status, lim); }, E, a.p,
+                                        a.rule, want_rank, sel_sc, a.status, &on, &r, &g);
             const int j = tid;
             if (j < E) {
                 const float gv = on ? (a.gate == PP_GATE_NONE ? 1.0f : sigmoidf_(g)) : 0.0f;
@@ -183,10 +198,9 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
                     mask[j] |= 1u << t;
                 }
                 if (publish) {
-                    if (a.sel_ids) {  // ranks are a permutation: every rank slot is written once
-                        a.sel_ids[(size_t)t * E + r] = on ? j : -1;
-                        a.sel_gates[(size_t)t * E + r] = gv;
-                    }
+                    if (a.sel_ids)
+                        write_selection_row(a.sel_ids + (size_t)t * E, a.sel_gates + (size_t)t * E, j, E, k, on, r,
+                                            gv);
                     if (a.sel_logits) a.sel_logits[(size_t)t * E + j] = g;
                 }
             }
@@ -231,7 +245,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     const int nt_w = ntiles > warp ? (ntiles - warp + kWarps - 1) / kWarps : 0;
     const int ded6 = a.ded6, slots6 = a.slots6;
     // a warp's first ded6 slots are its own part of the phase-6 ring; the
-    // others are carved from the phase-4 ring, free after the second barrier
+    // others are carved from the phase-4 ring, free once this CTA's phase 4
+    // is done
     auto slot6 = [&](int s) -> unsigned char* {
         return s < ded6 ? ring6 + (size_t)(warp * ded6 + s) * stage6
                         : ring4 + (size_t)(warp * (slots6 - ded6) + (s - ded6)) * stage6;
@@ -300,7 +315,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
         const int q = nb + i;
         const int u = q >> 6, n = q & 63;
         const float w = gw[t * E + ulist[u]];
-        a.h_ws[((size_t)u * T + t) * kDExpert + n] = w == 0.0f ? 0.0f : act_h(a.act, su, sg) * w;
+        st_tagged(a.th + ((size_t)u * T + t) * kDExpert + n, tag, w == 0.0f ? 0.0f : act_h(a.act, su, sg) * w);
     };
     // Few neurons (cnt <= NS4): all loads at once, neuron i -> slot i, each
     // neuron split into S column slices worked on by S warps.  Many neurons:
@@ -370,25 +385,15 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
         }
     }
 
-    grid_barrier(a.bar, a.status, lim);
+    // this CTA's phase-4 slots are free again (extra phase-6 slots below)
+    __syncthreads();
 
     // ---------------------------------------------------------- phase 6
     if (rows == 0) return;
-    // h of the first chunk of U -> shared memory (after the extra tile slots)
-    float* hs = reinterpret_cast<float*>(ring4 + (size_t)kWarps * (slots6 - ded6) * stage6);
-    const int uch = a.uch;  // experts per h chunk, a multiple of 8
-    const uint32_t hbytes_per_u = (uint32_t)(T * kDExpert * 4);
-    if (tid == 0 && ntiles > 0) {
-        fence_proxy_async_smem();
-        const uint32_t nbytes = (uint32_t)min(uch, ntiles) * hbytes_per_u;
-        mbar_arrive_expect_tx(&bars[kBarH], nbytes);
-        bulk_g2s(hs, a.h_ws, nbytes, &bars[kBarH]);
-    }
     if (lane == 0) {
         fence_proxy_async_smem();
         for (int i = ded6; i < min(nt_w, slots6); i++) issue6(i);
     }
-    if (ntiles > 0) mbar_wait(&bars[kBarH], 0, a.status, lim);
 
     // lane: chunk column c of the 64-wide block (8 elements; fp32 uses two
     // 4-element chunks c and c + 8) and rows rig + 4 j
@@ -399,43 +404,63 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     for (int j = 0; j < RPL; j++)
 #pragma unroll
         for (int t = 0; t < TS; t++) acc[j][t] = 0.0f;
-    const int nt_all = (ntiles + kWarps - 1) / kWarps;  // same trip count in every warp
-    int hchunk = 0;
-    for (int i = 0; i < nt_all; i++) {
+    // h of this warp's experts, hch experts at a time: bulk copies of their
+    // tagged words (written by the CTAs that own the experts' neurons) into
+    // the warp's part of the h area, repeated until every word carries this
+    // launch's tag
+    const int hch = a.hch;
+    const int hwords = T * kDExpert;  // h words of one expert slot
+    unsigned long long* hs_w =
+        reinterpret_cast<unsigned long long*>(ring4 + (size_t)kWarps * (slots6 - ded6) * stage6) +
+        (size_t)warp * hch * hwords;
+    uint64_t* hbar = &bars[kBarH + warp];
+    uint32_t hphase = 0;
+    for (int i = 0; i < nt_w; i++) {
         const int u = warp + kWarps * i;
-        if (kWarps * i >= (hchunk + 1) * uch) {  // next h chunk (uniform over the CTA)
-            __syncthreads();
-            hchunk++;
-            if (tid == 0) {
-                fence_proxy_async_smem();
-                const uint32_t nbytes = (uint32_t)min(uch, ntiles - hchunk * uch) * hbytes_per_u;
-                mbar_arrive_expect_tx(&bars[kBarH], nbytes);
-                bulk_g2s(hs, a.h_ws + (size_t)hchunk * uch * T * kDExpert, nbytes, &bars[kBarH]);
-            }
-            mbar_wait(&bars[kBarH], (uint32_t)hchunk & 1u, a.status, lim);
+        if (i % hch == 0) {
+            const int nc = min(hch, nt_w - i);
+            const int npairs = nc * hwords / 2;
+            uint64_t t0 = 0;
+            bool ready;
+            do {
+                __syncwarp();  // earlier reads of the area are done
+                if (lane == 0) {
+                    fence_proxy_async_smem();
+                    mbar_arrive_expect_tx(hbar, (uint32_t)(nc * hwords * 8));
+                    for (int ti = 0; ti < nc; ti++)
+                        bulk_g2s(hs_w + (size_t)ti * hwords, a.th + (size_t)(u + kWarps * ti) * hwords,
+                                 (uint32_t)(hwords * 8), hbar);
+                }
+                mbar_wait(hbar, hphase & 1u, a.status, lim);
+                hphase++;
+                ready = true;
+                for (int q = lane; q < npairs; q += 32) {
+                    const ulonglong2 w2 = reinterpret_cast<const ulonglong2*>(hs_w)[q];
+                    ready = ready && word_tag(w2.x) == tag && word_tag(w2.y) == tag;
+                }
+                ready = __all_sync(kFull, ready);
+                if (!ready) __nanosleep(kPollBackoffNs);
+            } while (!ready && !__shfl_sync(kFull, (int)poll_give_up(t0, a.status, lim), 0));
         }
-        if (i >= nt_w) continue;
-        const int s = i % slots6;
-        mbar_wait(&bars[kBarFull6 + warp * kMaxSlots6 + s], (uint32_t)(i / slots6) & 1u, a.status, lim);
-        const TW* tile = reinterpret_cast<const TW*>(slot6(s));
-        const float* hu = hs + (size_t)(u - hchunk * uch) * T * kDExpert;
+        const unsigned long long* hu = hs_w + (size_t)(i % hch) * hwords;
         float hv[TS][kCPL * kEl];
 #pragma unroll
         for (int t = 0; t < TS; t++)
             if (t < T)
 #pragma unroll
                 for (int cc = 0; cc < kCPL; cc++) {
-                    const float4* h4 =
-                        reinterpret_cast<const float4*>(hu + (size_t)t * kDExpert + (c + 8 * cc) * kEl);
+                    const ulonglong2* h2 =
+                        reinterpret_cast<const ulonglong2*>(hu + (size_t)t * kDExpert + (c + 8 * cc) * kEl);
 #pragma unroll
-                    for (int q4 = 0; q4 < kEl / 4; q4++) {
-                        const float4 v = h4[q4];
-                        hv[t][cc * kEl + q4 * 4 + 0] = v.x;
-                        hv[t][cc * kEl + q4 * 4 + 1] = v.y;
-                        hv[t][cc * kEl + q4 * 4 + 2] = v.z;
-                        hv[t][cc * kEl + q4 * 4 + 3] = v.w;
+                    for (int q2 = 0; q2 < kEl / 2; q2++) {
+                        const ulonglong2 v = h2[q2];
+                        hv[t][cc * kEl + q2 * 2 + 0] = word_value(v.x);
+                        hv[t][cc * kEl + q2 * 2 + 1] = word_value(v.y);
                     }
                 }
+        const int s = i % slots6;
+        mbar_wait(&bars[kBarFull6 + warp * kMaxSlots6 + s], (uint32_t)(i / slots6) & 1u, a.status, lim);
+        const TW* tile = reinterpret_cast<const TW*>(slot6(s));
 #pragma unroll
         for (int j = 0; j < RPL; j++) {
             const int row = rig + 4 * j;
@@ -521,20 +546,20 @@ bool decode_plan(const DecodePlanIn& in, DecodePlan* out) {
     if (off + stage4 > budget) return false;
     const size_t avail = budget - off;
     const int ns4 = (int)std::min<size_t>(kMaxNS4, avail / stage4);
-    // the ring also holds this CTA's router rows (phase 1) and, after phase
-    // 4, the extra phase-6 slots plus an h chunk of at least 8 experts
-    const size_t hper = (size_t)TS * kDExpert * 4;
+    // the ring also holds this CTA's router rows (phase 1) and, once phase 4
+    // is done, the extra phase-6 slots plus at least one expert's h per warp
+    const size_t hper = (size_t)TS * kDExpert * 8;  // tagged h words of one expert
     size_t ring4 = 0;
     int ext = kMaxSlots6 - p.ded6;
     for (; ext >= 0; ext--) {
         ring4 = std::max({(size_t)ns4 * stage4, (size_t)rpc * in.d * esz,
-                          (size_t)ext * kWarps * stage6 + 8 * hper});
+                          (size_t)ext * kWarps * stage6 + kWarps * hper});
         if (ring4 <= avail) break;
     }
     if (ext < 0) return false;
     p.slots6 = p.ded6 + ext;
     const size_t harea = ring4 - (size_t)ext * kWarps * stage6;
-    p.uch = (int)(std::min<size_t>(kMaxExperts, harea / hper) / 8 * 8);
+    p.hch = (int)std::min<size_t>((kMaxExperts + kWarps - 1) / kWarps, harea / (kWarps * hper));
     p.NS4 = ns4;
     p.smem = off + ring4;
     p.threads = kDecThreads;
@@ -575,6 +600,7 @@ static cudaError_t launch_rpl(const DecodeArgs& a, const DecodePlan& p, int grid
 
 cudaError_t decode_launch(const DecodeArgs& a, const DecodePlan& p, int dtype, int TS, int grid,
                           cudaStream_t st) {
+    if (grid < 1 || grid > kMaxGrid) return cudaErrorInvalidValue;  // one launch count per CTA
     if (dtype == PP_BF16) {
         switch (TS) {
             case 1: return launch_rpl<__nv_bfloat16, 1>(a, p, grid, st);

@@ -163,13 +163,11 @@ __global__ void __launch_bounds__(256) select_part_cta_kernel(const float* __res
     bool on;
     int r;
     float g;
-    const int k = cta_select_fn(load, E, p, rule, sc, status, &on, &r, &g);
+    const int k = cta_select_fn(load, E, p, rule, true, sc, status, &on, &r, &g);
     const int j = threadIdx.x;
-    if (j < E) {  // ranks are a permutation: every rank slot is written once
-        ids[(size_t)t * E + r] = on ? j : -1;
-        gates[(size_t)t * E + r] = on ? (gate == PP_GATE_NONE ? 1.0f : sigmoidf_(g)) : 0.0f;
-        if (logits_out) logits_out[(size_t)t * E + j] = g;
-    }
+    write_selection_row(ids + (size_t)t * E, gates + (size_t)t * E, j, E, k, on, r,
+                        on ? (gate == PP_GATE_NONE ? 1.0f : sigmoidf_(g)) : 0.0f);
+    if (j < E && logits_out) logits_out[(size_t)t * E + j] = g;
     if (j == 0) counts[t] = k;
 }
 

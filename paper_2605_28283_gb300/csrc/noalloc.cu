@@ -6,10 +6,11 @@
 // its own pool, a real-time loop that must not take the implicit device
 // synchronisation an allocation can cause, or a plug-in host that exposes no
 // allocation API to the code it loads.  This entry point runs the same fused
-// decode kernel as pp_layer, but its scratch memory (status word, grid
-// barrier counter, router logits and the gate/up activations) lives in one
-// file-scope device array that every GPU loading the library reserves until
-// the process exits.  Nothing is allocated or freed per call.
+// decode kernel as pp_layer, but its scratch memory (status word, per-CTA
+// launch counts, and the tagged router logits and
+// gate/up activations the CTAs hand to each other) lives in one file-scope
+// device array that every GPU loading the library reserves until the
+// process exits.  Nothing is allocated or freed per call.
 #include <cstring>
 #include <mutex>
 
@@ -20,10 +21,11 @@ namespace {
 
 // Limits of the no-allocation variant: up to 4 tokens per call, E <= 256.
 constexpr int kNoAllocMaxTokens = 4;
-constexpr size_t kCtlBytes = 256;  // status word + grid barrier counters (pp::Control)
-constexpr size_t kLogitBytes = (size_t)kNoAllocMaxTokens * pp::kMaxExperts * 4;
-constexpr size_t kHBytes = (size_t)pp::kMaxExperts * kNoAllocMaxTokens * pp::kDExpert * 4;
-constexpr size_t kScratchBytes = kCtlBytes + kLogitBytes + kHBytes;  // 266,496 bytes
+constexpr size_t kCtlBytes = sizeof(pp::Control);  // status word, per-CTA launch counts
+constexpr size_t kLogitBytes = (size_t)kNoAllocMaxTokens * pp::kMaxExperts * 8;
+constexpr size_t kHBytes = (size_t)pp::kMaxExperts * kNoAllocMaxTokens * pp::kDExpert * 8;
+constexpr size_t kScratchBytes = kCtlBytes + kLogitBytes + kHBytes;  // 533,760 bytes
+static_assert(kScratchBytes == 533760, "scratch size as documented in prunepath.h");
 constexpr uint64_t kTimeoutNs = 2000000000ull;
 
 }  // namespace
@@ -131,7 +133,7 @@ extern "C" pp_status pp_layer_noalloc(const pp_desc* desc, const void* x, int T,
     while (TS < T) TS <<= 1;
     pp::DecodePlan plan;
     const pp::DecodePlanIn in{d.dtype, d.d_model, d.n_experts, TS, ds->sms, d.act == PP_ACT_SWIGLU,
-                              ds->smem_optin - 4096};
+                              ds->smem_optin - pp::kDecodeStaticSmemReserve};
     if (!pp::decode_plan(in, &plan)) return PP_ERR_SHAPE;
 
     pp::DecodeArgs a;
@@ -150,10 +152,10 @@ extern "C" pp_status pp_layer_noalloc(const pp_desc* desc, const void* x, int T,
         a.sel_gates = sel_out->gates;
         a.sel_logits = sel_out->logits;
     }
-    a.logit_ws = reinterpret_cast<float*>(scratch + kCtlBytes);
-    a.h_ws = reinterpret_cast<float*>(scratch + kCtlBytes + kLogitBytes);
+    a.tlog = reinterpret_cast<unsigned long long*>(scratch + kCtlBytes);
+    a.th = reinterpret_cast<unsigned long long*>(scratch + kCtlBytes + kLogitBytes);
+    a.epochs = ctl->epoch;
     a.status = &ctl->status;
-    a.bar = &ctl->grid_bar[0];
     a.timeout_ns = kTimeoutNs;
     a.T = T;
     a.d = d.d_model;
@@ -168,7 +170,7 @@ extern "C" pp_status pp_layer_noalloc(const pp_desc* desc, const void* x, int T,
     a.NS4 = plan.NS4;
     a.ded6 = plan.ded6;
     a.slots6 = plan.slots6;
-    a.uch = plan.uch;
+    a.hch = plan.hch;
     a.off_x = plan.off_x;
     a.off_gw = plan.off_gw;
     a.off_mask = plan.off_mask;
@@ -178,9 +180,9 @@ extern "C" pp_status pp_layer_noalloc(const pp_desc* desc, const void* x, int T,
     a.off_ring6 = plan.off_ring6;
     a.off_ring4 = plan.off_ring4;
 
-    // The status word and the grid barrier counter must start at zero; the
-    // logits and activations are fully written before they are read.
-    if (cudaMemsetAsync(scratch, 0, kCtlBytes, st) != cudaSuccess) return PP_ERR_CUDA;
+    // The status word starts at zero for every call.  The launch counts and the tagged words carry over from call to
+    // call (zero at load time): a call only accepts words tagged by itself.
+    if (cudaMemsetAsync(&ctl->status, 0, sizeof(unsigned), st) != cudaSuccess) return PP_ERR_CUDA;
     if (pp::decode_launch(a, plan, d.dtype, TS, ds->sms, st) != cudaSuccess) return PP_ERR_CUDA;
     if (status_out &&
         cudaMemcpyAsync(status_out, &ctl->status, sizeof(uint32_t), cudaMemcpyDeviceToDevice, st) != cudaSuccess)

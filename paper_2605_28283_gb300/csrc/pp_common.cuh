@@ -1,8 +1,9 @@
 // Device helpers shared by the PrunePath kernels (sm_103a).
 //
 // Inline PTX wrappers for mbarriers, bulk and tensor TMA copies, proxy
-// fences and the global timer; a bounded mbarrier wait; a self-resetting
-// grid barrier for cooperative (co-resident) grids; bf16 helpers.
+// fences and the global timer; a bounded mbarrier wait; tagged 64-bit words
+// for handing values between the CTAs of one co-resident (cooperative) grid
+// without a grid barrier; bf16 helpers.
 #pragma once
 
 #include <cuda.h>
@@ -22,14 +23,15 @@ constexpr int kMaxD = 8192;
 constexpr unsigned kFull = 0xffffffffu;
 
 // ------------------------------------------------------------------ control
-// The first 256 bytes of every workspace.
+// The first 1280 bytes of every workspace.
+constexpr int kMaxGrid = 256;  // CTAs of a fused decode launch (one per SM)
 struct Control {
-    unsigned status;      // sticky pp_status of the device side
-    unsigned wait_flag;   // never written: target of pp_debug_wait_timeout
-    unsigned grid_bar[4]; // self-resetting grid barrier counters
-    unsigned pad[58];
+    unsigned status;           // sticky pp_status of the device side
+    unsigned wait_flag;        // never written: target of pp_debug_wait_timeout
+    unsigned pad[62];
+    unsigned epoch[kMaxGrid];  // launches of the fused decode kernel seen by CTA b
 };
-static_assert(sizeof(Control) == 256, "control block is 256 bytes");
+static_assert(sizeof(Control) == 1280, "control block is 1280 bytes");
 
 PP_DEVINL void record_status(unsigned* status, pp_status s) {
     // first error wins; later ones do not overwrite it
@@ -126,36 +128,70 @@ PP_DEVINL void named_bar_sync(int id, int nthreads) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
-// ------------------------------------------------------------ grid barrier
+// ---------------------------------------------------------- tagged words
 PP_DEVINL unsigned ld_acquire_gpu(const unsigned* p) {
     unsigned v;
     asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
 
-// Barrier across all CTAs of a co-resident (cooperative) grid.  The counter
-// returns to its starting value after every complete barrier, so one zeroed
-// word serves any number of barriers and launches.  Every thread of every
-// CTA must call it.  Bounded: after limit_ns the waiting CTA records
-// PP_ERR_TIMEOUT and continues.
-PP_DEVINL void grid_barrier(unsigned* counter, unsigned* status, uint64_t limit_ns) {
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        const unsigned nblocks = gridDim.x * gridDim.y * gridDim.z;
-        const bool first = (blockIdx.x | blockIdx.y | blockIdx.z) == 0;
-        const unsigned add = first ? (0x80000000u - (nblocks - 1u)) : 1u;
-        __threadfence();
-        const unsigned old = atomicAdd(counter, add);
-        const uint64_t t0 = globaltimer_ns();
-        while (((ld_acquire_gpu(counter) ^ old) & 0x80000000u) == 0u) {
-            if (globaltimer_ns() - t0 > limit_ns) {
-                record_status(status, PP_ERR_TIMEOUT);
-                break;
-            }
-        }
-        __threadfence();
+// A value handed from one CTA to others of the same launch travels with the
+// launch's tag in one 64-bit word, (tag << 32) | bits(value).  A 64-bit store
+// is single-copy atomic, so a reader that sees the tag sees the value: no
+// flag, fence or grid barrier is needed, and each reader waits only for the
+// words it uses.  Tags change from launch to launch (a launch never takes its
+// predecessor's words for current) and are not 0, the value of a zeroed
+// workspace, before 2^32 - 1 launches.
+PP_DEVINL void st_tagged(unsigned long long* p, unsigned tag, float v) {
+    const unsigned long long w = ((unsigned long long)tag << 32) | __float_as_uint(v);
+    asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(w) : "memory");
+}
+
+PP_DEVINL unsigned long long ld_relaxed_u64(const unsigned long long* p) {
+    unsigned long long v;
+    asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+
+PP_DEVINL void ld_relaxed_v2(const unsigned long long* p, unsigned long long& a, unsigned long long& b) {
+    asm volatile("ld.relaxed.gpu.global.v2.u64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "l"(p) : "memory");
+}
+
+PP_DEVINL unsigned word_tag(unsigned long long w) { return (unsigned)(w >> 32); }
+PP_DEVINL float word_value(unsigned long long w) { return __uint_as_float((unsigned)w); }
+
+// Pause between two polls of the same words: without it, every SM re-reading
+// a handful of L2 lines back to back slows the stores and loads of the CTAs
+// that are still working.
+constexpr unsigned kPollBackoffNs = 64;
+
+// Bookkeeping of a bounded poll: true when the caller should stop polling,
+// after limit_ns (recording PP_ERR_TIMEOUT) or, past 1 ms, as soon as another
+// wait has recorded an error.
+PP_DEVINL bool poll_give_up(uint64_t& t0, unsigned* status, uint64_t limit_ns) {
+    const uint64_t now = globaltimer_ns();
+    if (t0 == 0) {
+        t0 = now;
+        return false;
     }
-    __syncthreads();
+    const uint64_t dt = now - t0;
+    if (dt > limit_ns) {
+        record_status(status, PP_ERR_TIMEOUT);
+        return true;
+    }
+    return dt > 1000000ull && *reinterpret_cast<volatile unsigned*>(status) != 0u;
+}
+
+// Value of the tagged word at p once it carries `tag` (bounded; on giving up
+// the stale value is returned and the status says why).
+PP_DEVINL float wait_tagged(const unsigned long long* p, unsigned tag, unsigned* status, uint64_t limit_ns) {
+    unsigned long long w = ld_relaxed_u64(p);
+    uint64_t t0 = 0;
+    while (word_tag(w) != tag && !poll_give_up(t0, status, limit_ns)) {
+        __nanosleep(kPollBackoffNs);
+        w = ld_relaxed_u64(p);
+    }
+    return word_value(w);
 }
 
 // ------------------------------------------------------------------- bf16

@@ -26,16 +26,16 @@ struct DecodeArgs {
     int32_t* sel_counts;
     float* sel_gates;
     float* sel_logits;     // route: optional output
-    float* logit_ws;       // [T][E] scratch
-    float* h_ws;           // [|U|][T][64] scratch
+    unsigned long long* tlog;  // [T][E] tagged logits
+    unsigned long long* th;    // [|U|][T][64] tagged gate/up activations
+    unsigned* epochs;          // [grid] launch count per CTA (Control.epoch)
     unsigned* status;
-    unsigned* bar;
     uint64_t timeout_ns;
     int T, d, E;
     int act, gate, rule;
     float p;
     int do_route, do_ffn;
-    int R6, NS4, ded6, slots6, uch;
+    int R6, NS4, ded6, slots6, hch;
     uint32_t off_x, off_gw, off_mask, off_ulist, off_red, off_red6, off_ring6, off_ring4;
 };
 
@@ -46,10 +46,15 @@ struct DecodePlanIn {
 };
 
 struct DecodePlan {
-    int R6, RPL, NS4, ded6, slots6, uch, threads;
+    int R6, RPL, NS4, ded6, slots6, hch, threads;
     size_t smem;
     uint32_t off_x, off_gw, off_mask, off_ulist, off_red, off_red6, off_ring6, off_ring4;
 };
+
+// Part of the per-block shared-memory limit left to the decode kernel's
+// static shared memory (selection scratch and counters, 4 KB once padded to
+// the 1 KB alignment of the dynamic area).
+constexpr size_t kDecodeStaticSmemReserve = 6144;
 
 bool decode_plan(const DecodePlanIn& in, DecodePlan* out);
 cudaError_t decode_launch(const DecodeArgs& a, const DecodePlan& p, int dtype, int TS, int grid,

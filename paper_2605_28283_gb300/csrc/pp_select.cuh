@@ -147,21 +147,28 @@ PP_DEVINL float gate_of(int gate_mode, unsigned long long k) {
 // ---------------------------------------------------------------------------
 // CTA-parallel selection of one token (used where a single token's latency
 // matters).  Thread j owns expert j (E <= blockDim.x <= 256).  Instead of
-// sorting, every thread counts the experts ranked ahead of it (larger logit,
-// or equal logit and lower index) and sums their exponentials: its rank r_j
-// and the exclusive prefix mass S_{r_j - 1} in rank order.  The exponentials
-// e_j = exp(g_j - max g) (fp32) are summed as exact 2^-31 fixed-point
-// integers, and the cut compares S against p * Z exactly in integers, so
-// the only rounding is that of the fp32 exponentials.
-//   MIN_PREFIX: j activated <=> r_j == 0  or  S_{r_j - 1} <  p Z
-//   PAPER:      j activated <=> r_j == 0  or  S_{r_j}     <  p Z
-// (S non-decreasing along the order, so both are prefixes of the order.)
+// sorting, every thread sums the exponentials of the experts ranked ahead of
+// it: A_j = S_{r_j - 1}, the exclusive prefix mass at its rank r_j in the
+// descending order, with equal logits ordered by index: expert i is ahead
+// of j when its order key D_i (32 bits, smaller for a larger logit) is below
+// D_j, or equal to it with i < j.  Candidates of lower index are compared
+// with D_j + 1 and the others with D_j, so the count loop stays in 32-bit
+// compares.  The
+// exponentials e_j = exp(g_j - max g) (fp32) are summed as exact 2^-31
+// fixed-point integers and the cut compares masses with p * Z exactly in
+// integers, so the only rounding is that of the fp32 exponentials.
+//   MIN_PREFIX: j activated <=> A_j == 0 (rank 0)  or  A_j       <  p Z
+//   PAPER:      j activated <=> A_j == 0 (rank 0)  or  A_j + U_j <  p Z
+// (the top expert has e = 1, U = 2^31 > 0, so A_j == 0 exactly at rank 0;
+// A is non-decreasing along the order, so both sets are prefixes of it).
 
 struct CtaSelScratch {
-    uint32_t D[kMaxExperts];  // descending-order keys (smaller = larger logit)
-    uint32_t U[kMaxExperts];  // fixed-point exponentials, e * 2^31
+    // order keys D[0..255] and fixed-point exponentials U[256..511] (e * 2^31);
+    // after the count, the same bytes hold the activated (D, index) keys
+    __align__(16) uint32_t DU[2 * kMaxExperts];
     float fred[8];
     unsigned long long ured[8];
+    int wcnt[8];
 };
 
 PP_DEVINL uint32_t desc_key(float g) {
@@ -185,18 +192,20 @@ PP_DEVINL long long prefix_threshold(float p, unsigned long long Z) {
     return (long long)((rhs - 1ull) >> sh);
 }
 
-// Returns the activated count (CTA-uniform).  On return: *sel = whether
-// expert j (= threadIdx.x) is activated, *rank = its rank, *gval = its
-// logit.  All threads of the CTA (8 warps) must call it.
+// Returns the activated count k (CTA-uniform).  On return: *sel = whether
+// expert j (= threadIdx.x) is activated, *gval = its logit and, when
+// want_rank, *rank = its rank for activated experts (the activated experts
+// hold ranks 0 .. k-1); *rank is -1 otherwise.  All threads of the CTA (8
+// warps) must call it with the same want_rank.
 template <typename Load>
-PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, CtaSelScratch& sc, unsigned* status,
-                            bool* sel, int* rank, float* gval) {
+PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, bool want_rank, CtaSelScratch& sc,
+                            unsigned* status, bool* sel, int* rank, float* gval) {
     const int j = threadIdx.x;
     const int lane = j & 31, warp = j >> 5;
     const bool valid = j < E;
     const float g = valid ? load(j) : -INFINITY;
     *gval = g;
-    *rank = j;
+    *rank = -1;
     const bool fin = !valid || isfinite(g);
     if (!__syncthreads_and(fin)) {
         if (j == 0) record_status(status, PP_ERR_NONFINITE);
@@ -217,9 +226,11 @@ PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, CtaSelScratch& 
     // fixed-point exponentials and their sum Z
     const float e = valid ? expf(g - m) : 0.0f;
     const uint32_t U = valid ? __float2uint_rn(e * 2147483648.0f) : 0u;
-    const uint32_t D = valid ? desc_key(g) : 0xffffffffu;
-    sc.D[j] = D;
-    sc.U[j] = U;
+    const uint32_t D = valid ? desc_key(g) : 0xffffffffu;  // a finite logit never gives all ones
+    uint32_t* sD = sc.DU;
+    uint32_t* sU = sc.DU + kMaxExperts;
+    sD[j] = D;
+    sU[j] = U;
     unsigned long long z = U;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(kFull, z, o);
@@ -231,51 +242,88 @@ PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, CtaSelScratch& 
         const ulonglong2 a = v[0], b = v[1], c = v[2], d2 = v[3];
         Z = (a.x + a.y) + (b.x + b.y) + (c.x + c.y) + (d2.x + d2.y);
     }
-    // rank and exclusive prefix mass: experts with a strictly larger logit,
-    // four independent accumulator chains; equal logits are counted too and
-    // resolved by index afterwards (rare; equal logits have equal U)
-    int r0 = 0, r1 = 0, r2 = 0, r3 = 0, eq = 0;
+    // exclusive prefix mass: the exponentials of the experts ahead, four
+    // independent accumulator chains; candidates [0, w0) have a lower index
+    // than every thread of this warp, [w0, w1) are the warp's own experts,
+    // [w1, E) have a higher index
     unsigned long long m0 = 0, m1 = 0, m2 = 0, m3 = 0;
-    const int E4 = E & ~3;
-    for (int i = 0; i < E4; i += 4) {
-        const uint4 d4 = *reinterpret_cast<const uint4*>(&sc.D[i]);
-        const uint4 u4 = *reinterpret_cast<const uint4*>(&sc.U[i]);
-        r0 += d4.x < D; m0 += d4.x < D ? (unsigned long long)u4.x : 0ull; eq += d4.x == D;
-        r1 += d4.y < D; m1 += d4.y < D ? (unsigned long long)u4.y : 0ull; eq += d4.y == D;
-        r2 += d4.z < D; m2 += d4.z < D ? (unsigned long long)u4.z : 0ull; eq += d4.z == D;
-        r3 += d4.w < D; m3 += d4.w < D ? (unsigned long long)u4.w : 0ull; eq += d4.w == D;
+    const int w0 = warp * 32, w1 = min(E, w0 + 32);
+    if (w0 < E) {  // warps without an expert skip the count
+        const uint32_t thrB = D + 1u, thrA = D;
+        auto accum = [&](int i0, int i1, uint32_t th) {
+            int i = i0;
+#pragma unroll 4
+            for (; i + 4 <= i1; i += 4) {
+                const uint4 d4 = *reinterpret_cast<const uint4*>(&sD[i]);
+                const uint4 u4 = *reinterpret_cast<const uint4*>(&sU[i]);
+                m0 += d4.x < th ? (unsigned long long)u4.x : 0ull;
+                m1 += d4.y < th ? (unsigned long long)u4.y : 0ull;
+                m2 += d4.z < th ? (unsigned long long)u4.z : 0ull;
+                m3 += d4.w < th ? (unsigned long long)u4.w : 0ull;
+            }
+            for (; i < i1; i++) m0 += sD[i] < th ? (unsigned long long)sU[i] : 0ull;
+        };
+        accum(0, w0, thrB);
+        {  // the warp's own experts: lower index than j -> thrB, else thrA
+            int i = w0;
+#pragma unroll 2
+            for (; i + 4 <= w1; i += 4) {
+                const uint4 d4 = *reinterpret_cast<const uint4*>(&sD[i]);
+                const uint4 u4 = *reinterpret_cast<const uint4*>(&sU[i]);
+                m0 += d4.x < (i + 0 < j ? thrB : thrA) ? (unsigned long long)u4.x : 0ull;
+                m1 += d4.y < (i + 1 < j ? thrB : thrA) ? (unsigned long long)u4.y : 0ull;
+                m2 += d4.z < (i + 2 < j ? thrB : thrA) ? (unsigned long long)u4.z : 0ull;
+                m3 += d4.w < (i + 3 < j ? thrB : thrA) ? (unsigned long long)u4.w : 0ull;
+            }
+            for (; i < w1; i++) m0 += sD[i] < (i < j ? thrB : thrA) ? (unsigned long long)sU[i] : 0ull;
+        }
+        accum(w1, E, thrA);
     }
-    for (int i = E4; i < E; i++) {
-        r0 += sc.D[i] < D;
-        m0 += sc.D[i] < D ? (unsigned long long)sc.U[i] : 0ull;
-        eq += sc.D[i] == D;
-    }
-    int r = (r0 + r1) + (r2 + r3);
-    unsigned long long ahead_mass = (m0 + m1) + (m2 + m3);
-    if (valid && eq > 1) {  // ties: the equal logits of lower index are ahead
-        int tb = 0;
-        for (int i = 0; i < j; i++) tb += sc.D[i] == D ? 1 : 0;
-        r += tb;
-        ahead_mass += (unsigned long long)tb * U;
-    }
+    const unsigned long long ahead = (m0 + m1) + (m2 + m3);
     bool on;
     if (p >= 1.0f) {
         on = valid;
     } else {
         const long long thr = prefix_threshold(p, Z);
-        const unsigned long long mass = rule == PP_SEL_PAPER ? ahead_mass + U : ahead_mass;
-        on = valid && (r == 0 || (thr >= 0 && mass <= (unsigned long long)thr));
+        const unsigned long long mass = rule == PP_SEL_PAPER ? ahead + U : ahead;
+        on = valid && (ahead == 0ull || (thr >= 0 && mass <= (unsigned long long)thr));
     }
     *sel = on;
-    *rank = r;
-    return __syncthreads_count(on);
+    const int k = __syncthreads_count(on);  // also: every thread is done reading sD, sU
+    if (want_rank) {
+        // rank of an activated expert = activated keys (D, index) below its
+        // own; the activated keys are compacted into the scratch first
+        unsigned long long* sK = reinterpret_cast<unsigned long long*>(sc.DU);
+        const unsigned long long key = ((unsigned long long)D << 32) | (unsigned)j;
+        const unsigned bal = __ballot_sync(kFull, on);
+        if (lane == 0) sc.wcnt[warp] = __popc(bal);
+        __syncthreads();
+        int base = 0;
+        for (int w = 0; w < warp; w++) base += sc.wcnt[w];
+        if (on) sK[base + __popc(bal & ((1u << lane) - 1u))] = key;
+        __syncthreads();
+        if (on) {
+            int r = 0;
+            for (int i = 0; i < k; i++) r += sK[i] < key ? 1 : 0;
+            *rank = r;
+        }
+        __syncthreads();  // the scratch is reused by the next call
+    }
+    return k;
 }
 
-// Same, reading the logits (written by other CTAs earlier) from a row.
-PP_DEVINL int cta_select(const float* __restrict__ logits_row, int E, float p, int rule, CtaSelScratch& sc,
-                         unsigned* status, bool* sel, int* rank, float* gval) {
-    return cta_select_fn([&](int j) { return __ldcg(logits_row + j); }, E, p, rule, sc, status, sel, rank, gval);
+// The rank-order selection row of one token from cta_select_fn's results
+// (called by every thread j < E): activated experts at their ranks, -1 and
+// gate 0 in the slots k .. E-1.
+PP_DEVINL void write_selection_row(int32_t* ids, float* gates, int j, int E, int k, bool on, int r, float gv) {
+    if (on) {
+        ids[r] = j;
+        gates[r] = gv;
+    }
+    if (j >= k && j < E) {
+        ids[j] = -1;
+        gates[j] = 0.0f;
+    }
 }
-
 
 }  // namespace pp

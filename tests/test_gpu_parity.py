@@ -313,3 +313,42 @@ def test_deterministic(pp, T):
 def test_layer_f32_large_d(pp, d, T):
     """fp32 shapes whose x no longer fits 8 tokens per launch are sliced."""
     layer_parity(pp, "tiny_relu_f32", T, 0.7, d=d, E=16)
+
+
+def test_workspace_reuse_across_calls(pp):
+    """CTAs of the fused decode kernel hand logits and activations to each
+    other through tagged words that stay in the workspace between calls.  A
+    sequence of calls with changing token counts, p, entry points and a
+    re-initialisation on ONE workspace must give exactly what each call gives
+    on a fresh workspace (a stale word taken for current would change it)."""
+    import torch
+    w, L = layer_inputs("llama2_7b_decode", 4, d=1024, E=64)
+    desc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act)
+    x, Wr, Wg, Wu, Wd = (dev(a) for a in (L.x, L.Wr, L.Wg, L.Wu, L.Wd))
+    shared = pp.alloc_workspace(desc, 4)
+
+    def call(kind, T, p, ws):
+        sel = pp.Selection.empty(T, w.n_experts, "cuda")
+        y = torch.zeros((T, w.d_model), dtype=x.dtype, device="cuda")
+        if kind == "layer":
+            pp.pp_layer(desc, x[:T], T, Wr, Wg, Wu, Wd, p, sel, y, ws)
+        elif kind == "route":
+            pp.pp_route(desc, x[:T], T, Wr, p, sel, ws)
+        else:  # sparse FFN over the selection of the same tokens
+            pp.pp_route(desc, x[:T], T, Wr, p, sel, ws)
+            pp.pp_sparse_ffn(desc, x[:T], T, Wg, Wu, Wd, sel, y, ws)
+        torch.cuda.synchronize()
+        return to_host(sel.counts), to_host(sel.ids), to_host(y)
+
+    seq = [("layer", 4, 0.9), ("layer", 1, 0.3), ("route", 2, 0.7), ("layer", 3, 1.0), ("ffn", 2, 0.5),
+           ("layer", 1, 0.0), ("layer", 4, 0.7), ("init", 0, 0), ("layer", 2, 0.9), ("layer", 2, 0.9)]
+    for kind, T, p in seq:
+        if kind == "init":
+            pp.pp_workspace_init(shared)
+            continue
+        pf = f32(p)
+        got = call(kind, T, pf, shared)
+        want = call(kind, T, pf, pp.alloc_workspace(desc, 4))
+        for a, b in zip(got, want):
+            assert np.array_equal(a, b), (kind, T, p)
+        assert pp.pp_get_device_status(shared) == pp.PP_OK
