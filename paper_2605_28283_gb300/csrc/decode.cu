@@ -18,8 +18,8 @@
 //   phase 6  down projection: CTA b owns R6 rows of W_down and y.  Warp w
 //            handles the experts u = w, w+8, ... of U: it streams the
 //            [R6 x 64] column block of each with 2-D tensor TMA into its own
-//            slots (the first ones are issued before phase 4, so they
-//            overlap it), waits for those experts' h words and accumulates
+//            slots (issued as its phase 4 ends, so that they overlap the h
+//            exchange), waits for those experts' h words and accumulates
 //            every row of the CTA in registers; one cross-warp reduction in
 //            shared memory then writes y once (no atomics: deterministic).
 // There is no grid barrier: a CTA waits only for the words it reads.  Each
@@ -319,9 +319,9 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     };
     // Few neurons (cnt <= NS4): all loads at once, neuron i -> slot i, each
     // neuron split into S column slices worked on by S warps.  Many neurons:
-    // warp w streams neurons w, w + NS4, ... through slot w.  The phase-4
-    // loads go into the copy queue before the phase-6 prefetch.
+    // warp w streams neurons w, w + NS4, ... through slot w.
     const bool few = cnt > 0 && cnt <= a.NS4;
+    const int S = cnt == 1 ? 8 : cnt == 2 ? 4 : cnt <= 4 ? 2 : 1;
     if (few && tid == 0) {
         fence_proxy_async_smem();
         for (int i = 0; i < cnt; i++) issue4(i, i);
@@ -330,13 +330,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
         fence_proxy_async_smem();
         issue4(warp, warp);
     }
-    __syncwarp();
-    if (lane == 0) {
-        fence_proxy_async_smem();
-        for (int i = 0; i < min(nt_w, ded6); i++) issue6(i);  // phase-6 prefetch
-    }
     if (few) {
-        const int S = cnt == 1 ? 8 : cnt == 2 ? 4 : cnt <= 4 ? 2 : 1;
         if (warp < cnt * S) {
             const int i = warp / S, sl = warp % S;
             const int cs = (nchunk + S - 1) / S;
@@ -385,6 +379,14 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
         }
     }
 
+    // W_down tiles of phase 6: issued only now, so that across the grid the
+    // gate/up bytes that phase 4 waits for are not queued behind W_down bytes
+    // (the h exchange that phase 6 waits for anyway covers their latency)
+    __syncwarp();
+    if (lane == 0) {
+        fence_proxy_async_smem();
+        for (int i = 0; i < min(nt_w, ded6); i++) issue6(i);
+    }
     // this CTA's phase-4 slots are free again (extra phase-6 slots below)
     __syncthreads();
 

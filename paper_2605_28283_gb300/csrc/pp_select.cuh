@@ -250,34 +250,35 @@ PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, bool want_rank,
     const int w0 = warp * 32, w1 = min(E, w0 + 32);
     if (w0 < E) {  // warps without an expert skip the count
         const uint32_t thrB = D + 1u, thrA = D;
-        auto accum = [&](int i0, int i1, uint32_t th) {
+        // candidates [i0, i1) against threshold th (or, in the warp's own
+        // range, th for index >= j and th + 1 below j); 16 candidates are
+        // loaded before any of them is compared, so the shared-memory
+        // latency is paid once per 16
+        auto accum = [&](int i0, int i1, uint32_t th, bool own) {
             int i = i0;
-#pragma unroll 4
-            for (; i + 4 <= i1; i += 4) {
-                const uint4 d4 = *reinterpret_cast<const uint4*>(&sD[i]);
-                const uint4 u4 = *reinterpret_cast<const uint4*>(&sU[i]);
-                m0 += d4.x < th ? (unsigned long long)u4.x : 0ull;
-                m1 += d4.y < th ? (unsigned long long)u4.y : 0ull;
-                m2 += d4.z < th ? (unsigned long long)u4.z : 0ull;
-                m3 += d4.w < th ? (unsigned long long)u4.w : 0ull;
+            for (; i + 16 <= i1; i += 16) {
+                uint4 d4[4], u4[4];
+#pragma unroll
+                for (int k = 0; k < 4; k++) {
+                    d4[k] = *reinterpret_cast<const uint4*>(&sD[i + 4 * k]);
+                    u4[k] = *reinterpret_cast<const uint4*>(&sU[i + 4 * k]);
+                }
+#pragma unroll
+                for (int k = 0; k < 4; k++) {
+                    const int b = i + 4 * k;
+                    const uint32_t t0 = own && b + 0 < j ? th + 1u : th, t1 = own && b + 1 < j ? th + 1u : th;
+                    const uint32_t t2 = own && b + 2 < j ? th + 1u : th, t3 = own && b + 3 < j ? th + 1u : th;
+                    m0 += d4[k].x < t0 ? (unsigned long long)u4[k].x : 0ull;
+                    m1 += d4[k].y < t1 ? (unsigned long long)u4[k].y : 0ull;
+                    m2 += d4[k].z < t2 ? (unsigned long long)u4[k].z : 0ull;
+                    m3 += d4[k].w < t3 ? (unsigned long long)u4[k].w : 0ull;
+                }
             }
-            for (; i < i1; i++) m0 += sD[i] < th ? (unsigned long long)sU[i] : 0ull;
+            for (; i < i1; i++) m0 += sD[i] < (own && i < j ? th + 1u : th) ? (unsigned long long)sU[i] : 0ull;
         };
-        accum(0, w0, thrB);
-        {  // the warp's own experts: lower index than j -> thrB, else thrA
-            int i = w0;
-#pragma unroll 2
-            for (; i + 4 <= w1; i += 4) {
-                const uint4 d4 = *reinterpret_cast<const uint4*>(&sD[i]);
-                const uint4 u4 = *reinterpret_cast<const uint4*>(&sU[i]);
-                m0 += d4.x < (i + 0 < j ? thrB : thrA) ? (unsigned long long)u4.x : 0ull;
-                m1 += d4.y < (i + 1 < j ? thrB : thrA) ? (unsigned long long)u4.y : 0ull;
-                m2 += d4.z < (i + 2 < j ? thrB : thrA) ? (unsigned long long)u4.z : 0ull;
-                m3 += d4.w < (i + 3 < j ? thrB : thrA) ? (unsigned long long)u4.w : 0ull;
-            }
-            for (; i < w1; i++) m0 += sD[i] < (i < j ? thrB : thrA) ? (unsigned long long)sU[i] : 0ull;
-        }
-        accum(w1, E, thrA);
+        accum(0, w0, thrB, false);
+        accum(w0, w1, thrA, true);
+        accum(w1, E, thrA, false);
     }
     const unsigned long long ahead = (m0 + m1) + (m2 + m3);
     bool on;
