@@ -230,11 +230,13 @@ __global__ void __launch_bounds__(kDispBlock) dispatch_count_kernel(const uint32
 }
 
 // One block, thread e: hist, offsets (exclusive scan over experts), the
-// per-token-block bases and the expert's 128-row work items.
+// per-token-block bases and the expert's 128-row work items; clears the
+// overflow flag of the down projection.
 __global__ void __launch_bounds__(kMaxExperts) dispatch_scan_kernel(const int* __restrict__ blkcnt, int nblk, int E,
                                                                     int* offsets, int* blkbase, WorkItem* items,
-                                                                    int* n_items) {
+                                                                    int* n_items, int* overflow) {
     const int e = threadIdx.x;
+    if (e == 0) *overflow = 0;  // the down projection's overflow flag starts clear
     __shared__ int sh[kMaxExperts], si[kMaxExperts];
     int h = 0;
     if (e < E)
@@ -293,6 +295,133 @@ __global__ void __launch_bounds__(kDispBlock) dispatch_scatter_kernel(const uint
             perm_gate[pos] = gexp[(size_t)t * E + e];
             invpos[(size_t)t * E + e] = pos;
         }
+    }
+}
+
+// All of the dispatch for T <= 256 tokens in one CTA of 1024 threads (small
+// batches are latency-bound: four kernels with a serial loop over the
+// experts cost more than their work).  Shared memory holds, per expert, the
+// 256-bit mask of the tokens that activated it; an assignment (t, e) lands
+// at offsets[e] + (tokens below t in e's mask), so tokens stay in ascending
+// order within each expert, as in the multi-block path.  Writes the same
+// outputs as that path (bits, offsets, work items, perm_token, perm_gate,
+// invpos) and clears the overflow flag of the down projection.  Gates of a
+// repeated id add up (with three or more copies the order of the additions
+// is not fixed).
+constexpr int kSmallDispatchMaxT = 256;
+
+__global__ void __launch_bounds__(1024) dispatch_small_kernel(const int32_t* __restrict__ ids,
+                                                              const int32_t* __restrict__ counts,
+                                                              const float* __restrict__ gates, int T, int E,
+                                                              uint32_t* bits, int* offsets, WorkItem* items,
+                                                              int* n_items, int* perm_token, float* perm_gate,
+                                                              int* invpos, int* overflow, unsigned* status) {
+    __shared__ uint32_t mask[kMaxExperts][8];              // tokens of expert e
+    __shared__ uint32_t dup[kSmallDispatchMaxT][8];        // entry (t, r) repeats an earlier id of token t
+    __shared__ int off_s[kMaxExperts + 1], item_s[kMaxExperts + 1];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    for (int i = tid; i < kMaxExperts * 8; i += blockDim.x) {
+        (&mask[0][0])[i] = 0u;
+        (&dup[0][0])[i] = 0u;
+    }
+    if (tid == 0) *overflow = 0;
+    __syncthreads();
+    // token masks: warp w takes tokens w, w + 32, ...; lane r its entries
+    for (int t = warp; t < T; t += 32) {
+        int k = counts[t];
+        if (k < 0 || k > E) {
+            if (lane == 0) record_status(status, PP_ERR_INVALID_ARG);
+            k = k < 0 ? 0 : E;
+        }
+        for (int r = lane; r < k; r += 32) {
+            const int e = ids[(size_t)t * E + r];
+            if (e < 0 || e >= E) {
+                record_status(status, PP_ERR_INVALID_ARG);
+                continue;
+            }
+            const uint32_t bit = 1u << (t & 31);
+            if (atomicOr(&mask[e][t >> 5], bit) & bit) atomicOr(&dup[t][r >> 5], 1u << (r & 31));
+        }
+    }
+    __syncthreads();
+    // per-expert counts -> offsets and work items (warp 0 scans, 8 experts per lane)
+    if (warp == 0) {
+        int c[8], m[8], cs = 0, ms = 0;
+#pragma unroll
+        for (int q = 0; q < 8; q++) {
+            const int e = lane * 8 + q;
+            int n = 0;
+            if (e < E)
+#pragma unroll
+                for (int w = 0; w < 8; w++) n += __popc(mask[e][w]);
+            c[q] = n;
+            m[q] = (n + 127) >> 7;
+            cs += n;
+            ms += m[q];
+        }
+        int ci = cs, mi = ms;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int cv = __shfl_up_sync(kFull, ci, o), mv = __shfl_up_sync(kFull, mi, o);
+            if (lane >= o) {
+                ci += cv;
+                mi += mv;
+            }
+        }
+        int ce = ci - cs, me = mi - ms;
+#pragma unroll
+        for (int q = 0; q < 8; q++) {
+            off_s[lane * 8 + q] = ce;
+            item_s[lane * 8 + q] = me;
+            ce += c[q];
+            me += m[q];
+        }
+        if (lane == 31) {
+            off_s[kMaxExperts] = ci;
+            item_s[kMaxExperts] = mi;
+        }
+    }
+    __syncthreads();
+    if (tid < E) {
+        const int e = tid, o = off_s[e], n = off_s[e + 1] - o;
+        offsets[e] = o;
+        int it = item_s[e];
+        for (int a0 = 0; a0 < n; a0 += 128) items[it++] = WorkItem{e, o + a0, min(128, n - a0), 0};
+    }
+    if (tid == 0) {
+        offsets[E] = off_s[kMaxExperts];
+        *n_items = item_s[kMaxExperts];
+    }
+    // bits[t][w]: bit i of word w = token t activated expert 32 w + i
+    for (int q = tid; q < T * 8; q += blockDim.x) {
+        const int t = q >> 3, w = q & 7;
+        uint32_t v = 0;
+        for (int i = 0; i < 32 && 32 * w + i < E; i++) v |= ((mask[32 * w + i][t >> 5] >> (t & 31)) & 1u) << i;
+        bits[(size_t)t * 8 + w] = v;
+    }
+    // scatter: the first entry of each (t, e) writes its slot, repeats add
+    // their gate afterwards
+    for (int pass = 0; pass < 2; pass++) {
+        for (int t = warp; t < T; t += 32) {
+            const int k = min(max(counts[t], 0), E);
+            for (int r = lane; r < k; r += 32) {
+                const int e = ids[(size_t)t * E + r];
+                if (e < 0 || e >= E) continue;
+                const bool rep = (dup[t][r >> 5] >> (r & 31)) & 1u;
+                if (rep != (pass == 1)) continue;
+                int pos = off_s[e] + __popc(mask[e][t >> 5] & ((1u << (t & 31)) - 1u));
+                for (int w = 0; w < (t >> 5); w++) pos += __popc(mask[e][w]);
+                const float gv = gates[(size_t)t * E + r];
+                if (pass == 0) {
+                    perm_token[pos] = t;
+                    perm_gate[pos] = gv;
+                    invpos[(size_t)t * E + e] = pos;
+                } else {
+                    atomicAdd(&perm_gate[pos], gv);
+                }
+            }
+        }
+        __syncthreads();
     }
 }
 
@@ -570,50 +699,52 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 }
 
 // =================================================================== combine
-// One CTA per token: y[t] = (accumulator row, if any overflow) + the rows of
-// t's assignments in ascending expert order; fp32 sums, output bf16.
+// y[t] = the sum of token t's assignment rows Y[pos] in ascending expert
+// order, plus yacc[t] when the down projection overflowed (yacc is then
+// cleared again).  Grid (T, ceil(d / 1024)): 128 threads of 8 columns each.
+// The expert list is built in parallel: 128 experts per round, compacted in
+// ascending order with ballots.
 __global__ void __launch_bounds__(128) combine_kernel(const uint32_t* __restrict__ bits, const int* __restrict__ invpos,
                                                       const __nv_bfloat16* __restrict__ Y, long long ycap,
                                                       float* yacc, const int* __restrict__ overflow, int T, int E,
                                                       int d, __nv_bfloat16* y) {
-    const int t = blockIdx.x;
+    const int t = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     __shared__ int pos_s[kMaxExperts];
-    __shared__ int n_s;
-    if (threadIdx.x == 0) {
-        int n = 0;
-        for (int wdx = 0; wdx < 8; wdx++) {
-            uint32_t w = bits[(size_t)t * 8 + wdx];
-            while (w) {
-                const int e = wdx * 32 + __ffs(w) - 1;
-                w &= w - 1;
-                const int pos = invpos[(size_t)t * E + e];
-                if (pos < ycap) pos_s[n++] = pos;
-            }
-        }
-        n_s = n;
+    __shared__ int wn_s[4];
+    int n = 0;
+    for (int e0 = 0; e0 < E; e0 += 128) {
+        const int e = e0 + tid;
+        bool on = e < E && ((bits[(size_t)t * 8 + (e >> 5)] >> (e & 31)) & 1u);
+        const int pos = on ? invpos[(size_t)t * E + e] : 0;
+        on = on && pos < ycap;
+        const unsigned bal = __ballot_sync(kFull, on);
+        if (lane == 0) wn_s[warp] = __popc(bal);
+        __syncthreads();
+        int base = n;
+        for (int w = 0; w < warp; w++) base += wn_s[w];
+        if (on) pos_s[base + __popc(bal & ((1u << lane) - 1u))] = pos;
+        n += wn_s[0] + wn_s[1] + wn_s[2] + wn_s[3];
+        __syncthreads();
     }
-    __syncthreads();
-    const int n = n_s;
-    const bool ovf = *overflow != 0;
-    for (int c = threadIdx.x * 8; c < d; c += blockDim.x * 8) {
-        float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-        if (ovf) {
-            float4* ya = reinterpret_cast<float4*>(yacc + (size_t)t * d + c);
-            const float4 a0 = ya[0], a1 = ya[1];
-            acc[0] = a0.x; acc[1] = a0.y; acc[2] = a0.z; acc[3] = a0.w;
-            acc[4] = a1.x; acc[5] = a1.y; acc[6] = a1.z; acc[7] = a1.w;
-            ya[0] = make_float4(0.f, 0.f, 0.f, 0.f);  // keep the accumulator zero at rest
-            ya[1] = make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-        for (int i = 0; i < n; i++) {
-            const uint4 v = *reinterpret_cast<const uint4*>(Y + (size_t)pos_s[i] * d + c);
-            acc[0] += bf16lo(v.x); acc[1] += bf16hi(v.x); acc[2] += bf16lo(v.y); acc[3] += bf16hi(v.y);
-            acc[4] += bf16lo(v.z); acc[5] += bf16hi(v.z); acc[6] += bf16lo(v.w); acc[7] += bf16hi(v.w);
-        }
-        *reinterpret_cast<uint4*>(y + (size_t)t * d + c) =
-            make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]), pack_bf16x2(acc[4], acc[5]),
-                       pack_bf16x2(acc[6], acc[7]));
+    const int c = blockIdx.y * 1024 + tid * 8;
+    if (c >= d) return;
+    float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    if (*overflow != 0) {
+        float4* ya = reinterpret_cast<float4*>(yacc + (size_t)t * d + c);
+        const float4 a0 = ya[0], a1 = ya[1];
+        acc[0] = a0.x; acc[1] = a0.y; acc[2] = a0.z; acc[3] = a0.w;
+        acc[4] = a1.x; acc[5] = a1.y; acc[6] = a1.z; acc[7] = a1.w;
+        ya[0] = make_float4(0.f, 0.f, 0.f, 0.f);  // keep the accumulator zero at rest
+        ya[1] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
+    for (int i = 0; i < n; i++) {
+        const uint4 v = *reinterpret_cast<const uint4*>(Y + (size_t)pos_s[i] * d + c);
+        acc[0] += bf16lo(v.x); acc[1] += bf16hi(v.x); acc[2] += bf16lo(v.y); acc[3] += bf16hi(v.y);
+        acc[4] += bf16lo(v.z); acc[5] += bf16hi(v.z); acc[6] += bf16lo(v.w); acc[7] += bf16hi(v.w);
+    }
+    *reinterpret_cast<uint4*>(y + (size_t)t * d + c) =
+        make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]), pack_bf16x2(acc[4], acc[5]),
+                   pack_bf16x2(acc[6], acc[7]));
 }
 
 // ====================================================================== host
@@ -706,15 +837,20 @@ cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
     const bool gated = a.act == PP_ACT_SWIGLU;
     cudaError_t e;
     // dispatch
-    const int nblk = (a.T + kDispBlock - 1) / kDispBlock;
-    dispatch_bits_kernel<<<(a.T + 255) / 256, 256, 0, st>>>(a.ids, a.counts, a.gates, a.T, a.E, a.bits, a.gexp,
-                                                             a.status);
-    dispatch_count_kernel<<<nblk, kDispBlock, 0, st>>>(a.bits, a.T, a.E, a.wcnt, a.blkcnt);
-    dispatch_scan_kernel<<<1, kMaxExperts, 0, st>>>(a.blkcnt, nblk, a.E, a.offsets, a.blkbase,
-                                                   reinterpret_cast<WorkItem*>(a.items), a.n_items);
-    dispatch_scatter_kernel<<<nblk, kDispBlock, 0, st>>>(a.bits, a.gexp, a.T, a.E, a.wcnt, a.blkbase, a.perm_token,
-                                                        a.perm_gate, a.invpos);
-    if ((e = cudaMemsetAsync(a.overflow, 0, 4, st)) != cudaSuccess) return e;
+    if (a.T <= kSmallDispatchMaxT) {
+        dispatch_small_kernel<<<1, 1024, 0, st>>>(a.ids, a.counts, a.gates, a.T, a.E, a.bits, a.offsets,
+                                                  reinterpret_cast<WorkItem*>(a.items), a.n_items, a.perm_token,
+                                                  a.perm_gate, a.invpos, a.overflow, a.status);
+    } else {
+        const int nblk = (a.T + kDispBlock - 1) / kDispBlock;
+        dispatch_bits_kernel<<<(a.T + 255) / 256, 256, 0, st>>>(a.ids, a.counts, a.gates, a.T, a.E, a.bits,
+                                                                 a.gexp, a.status);
+        dispatch_count_kernel<<<nblk, kDispBlock, 0, st>>>(a.bits, a.T, a.E, a.wcnt, a.blkcnt);
+        dispatch_scan_kernel<<<1, kMaxExperts, 0, st>>>(a.blkcnt, nblk, a.E, a.offsets, a.blkbase,
+                                                       reinterpret_cast<WorkItem*>(a.items), a.n_items, a.overflow);
+        dispatch_scatter_kernel<<<nblk, kDispBlock, 0, st>>>(a.bits, a.gexp, a.T, a.E, a.wcnt, a.blkbase,
+                                                            a.perm_token, a.perm_gate, a.invpos);
+    }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     // grouped gate/up
     CUtensorMap mx1, mwg, mwu, mh, mwd;
@@ -746,8 +882,9 @@ cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
                                                          a.status, a.timeout_ns);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
-    combine_kernel<<<a.T, 128, 0, st>>>(a.bits, a.invpos, a.Y, g.ycap, a.yacc, a.overflow, a.T, a.E, a.d,
-                                        reinterpret_cast<__nv_bfloat16*>(a.y));
+    combine_kernel<<<dim3(a.T, (a.d + 1023) / 1024), 128, 0, st>>>(a.bits, a.invpos, a.Y, g.ycap, a.yacc,
+                                                                 a.overflow, a.T, a.E, a.d,
+                                                                 reinterpret_cast<__nv_bfloat16*>(a.y));
     return cudaGetLastError();
 }
 
