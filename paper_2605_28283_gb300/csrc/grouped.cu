@@ -93,24 +93,27 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         umma_commit(&tfull);
     } else if (warp >= 2) {
+        // lane = row 32 q + lane of the tile; 32 x 32 blocks are transposed
+        // through shared memory (the pipeline stages are free once every MMA
+        // has completed) so that each store writes 32 consecutive logits of
+        // one row
         const int q = warp & 3;
-        const int row = 32 * q + lane;
-        const int t = m0 + row;
         mbar_wait(&tfull, 0, status, lim);
         tc_fence_after();
-        float* dst = part + ((size_t)split * T + t) * E;
+        float* tr = reinterpret_cast<float*>(smem) + (size_t)(warp - 2) * 32 * 33;
 #pragma unroll 1
         for (int c = 0; c < NE; c += 32) {
             uint32_t r[32];
             tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)c, r);
             tmem_ld_wait();
-            if (t < T && k1 > k0)
 #pragma unroll
-                for (int i = 0; i < 32; i++)
-                    if (c + i < E) dst[c + i] = __uint_as_float(r[i]);
-            if (t < T && k1 <= k0)
-                for (int i = 0; i < 32; i++)
-                    if (c + i < E) dst[c + i] = 0.0f;
+            for (int i = 0; i < 32; i++) tr[lane * 33 + i] = k1 > k0 ? __uint_as_float(r[i]) : 0.0f;
+            __syncwarp();
+            for (int i = 0; i < 32; i++) {
+                const int t = m0 + 32 * q + i;
+                if (t < T && c + lane < E) part[((size_t)split * T + t) * E + c + lane] = tr[i * 33 + lane];
+            }
+            __syncwarp();
         }
     }
     tc_fence_before();
@@ -569,13 +572,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 PP_DEVINL bool jt_first_overflow(const WorkItem& w, long long ycap) { return (long long)w.a0 + w.cnt > ycap; }
 
 // ============================================================== grouped down
-// Persistent over work items; per item the H tile is loaded once and the
-// njt 256-wide slices of d stream through the B ring.  Two 256-column TMEM
-// accumulators overlap the reduction epilogue with the next slice's MMAs.
+// Persistent over (work item, column part) pairs: the njt 256-wide slices of
+// d are cut into nsub parts (more, smaller tasks than items when a batch is
+// small, so that every SM streams W_down); per task the H tile is loaded
+// once and the part's slices stream through the B ring.  Two 256-column
+// TMEM accumulators overlap the reduction epilogue with the next slice's
+// MMAs.
 __global__ void __launch_bounds__(kTcThreads, 1)
     down_gemm_kernel(const __grid_constant__ CUtensorMap map_h, const __grid_constant__ CUtensorMap map_wd,
                      const WorkItem* __restrict__ items, const int* __restrict__ n_items_p,
-                     const int* __restrict__ perm_token, int d, int njt, __nv_bfloat16* Y, long long ycap,
+                     const int* __restrict__ perm_token, int d, int njt, int nsub, __nv_bfloat16* Y, long long ycap,
                      float* yacc, int* overflow, unsigned* status, uint64_t lim) {
     constexpr int kStages = 4;
     constexpr int kTileB = 256 * 128;
@@ -586,7 +592,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     __shared__ uint64_t full[kStages], empty[kStages], tfull[2], tempty[2], afull, aempty;
     __shared__ uint32_t taddr_s;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n_items = *n_items_p;
+    const int n_tasks = *n_items_p * nsub;
+    // slices [jt0, jt1) of task v (item v / nsub, part v % nsub)
+    auto slices = [&](int v, int& jt0, int& jt1) {
+        const int sp = v % nsub;
+        jt0 = sp * njt / nsub;
+        jt1 = (sp + 1) * njt / nsub;
+    };
     if (threadIdx.x == 0) {
         for (int i = 0; i < kStages; i++) {
             mbar_init(&full[i], 1);
@@ -612,12 +624,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (warp == 0) {
         if (lane == 0) {
             int it = 0, ii = 0;
-            for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x, ii++) {
-                const WorkItem w = items[wi];
+            for (int v = blockIdx.x; v < n_tasks; v += gridDim.x, ii++) {
+                const WorkItem w = items[v / nsub];
+                int jt0, jt1;
+                slices(v, jt0, jt1);
                 if (ii >= 1) mbar_wait(&aempty, (uint32_t)(ii - 1) & 1u, status, lim);
                 mbar_arrive_expect_tx(&afull, kTileBytesA);
                 tma_load_2d(tileA, &map_h, 0, w.a0, &afull);
-                for (int jt = 0; jt < njt; jt++, it++) {
+                for (int jt = jt0; jt < jt1; jt++, it++) {
                     const int s = it % kStages;
                     if (it >= kStages) mbar_wait(&empty[s], (uint32_t)((it / kStages) - 1) & 1u, status, lim);
                     mbar_arrive_expect_tx(&full[s], kTileB);
@@ -630,9 +644,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (lane == 0) {
             constexpr uint32_t idesc = idesc_bf16_m128(256);
             int it = 0, acc = 0, ii = 0;
-            for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x, ii++) {
+            for (int v = blockIdx.x; v < n_tasks; v += gridDim.x, ii++) {
+                int jt0, jt1;
+                slices(v, jt0, jt1);
                 mbar_wait(&afull, (uint32_t)ii & 1u, status, lim);
-                for (int jt = 0; jt < njt; jt++, it++, acc++) {
+                for (int jt = jt0; jt < jt1; jt++, it++, acc++) {
                     const int a = acc & 1;
                     if (acc >= 2) mbar_wait(&tempty[a], (uint32_t)((acc >> 1) - 1) & 1u, status, lim);
                     const int s = it % kStages;
@@ -650,22 +666,25 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int q = warp & 3;
         const int row = 32 * q + lane;
         int acc = 0;
-        for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x) {
-            const WorkItem w = items[wi];
+        for (int v = blockIdx.x; v < n_tasks; v += gridDim.x) {
+            const WorkItem w = items[v / nsub];
+            int jt0, jt1;
+            slices(v, jt0, jt1);
             const bool live = row < w.cnt;
+            const bool group_live = 32 * q < w.cnt;  // any live row in this warp's 32 rows
             const long long arow = (long long)w.a0 + row;
             const bool in_buf = live && arow < ycap;
             const int tok = live && !in_buf ? perm_token[arow] : -1;
             float* yrow = tok >= 0 ? yacc + (size_t)tok * d : nullptr;
             if (tok >= 0 && jt_first_overflow(w, ycap)) *overflow = 1;
             __nv_bfloat16* Yrow = in_buf ? Y + (size_t)arow * d : nullptr;
-            for (int jt = 0; jt < njt; jt++, acc++) {
+            for (int jt = jt0; jt < jt1; jt++, acc++) {
                 const int a = acc & 1;
                 mbar_wait(&tfull[a], (uint32_t)(acc >> 1) & 1u, status, lim);
                 tc_fence_after();
                 const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(a * 256);
 #pragma unroll 1
-                for (int c = 0; c < 256; c += 32) {
+                for (int c = 0; c < (group_live ? 256 : 0); c += 32) {
                     uint32_t r[32];
                     tmem_ld32(base + (uint32_t)c, r);
                     tmem_ld_wait();
@@ -877,9 +896,14 @@ cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
     {
         const size_t smem = (size_t)kTileBytesA + 4 * (size_t)256 * 128 + 1024;
         if ((e = set_smem(down_gemm_kernel, smem)) != cudaSuccess) return e;
-        down_gemm_kernel<<<grid, kTcThreads, smem, st>>>(mh, mwd, items, a.n_items, a.perm_token, a.d,
-                                                         (a.d + 255) / 256, a.Y, g.ycap, a.yacc, a.overflow,
-                                                         a.status, a.timeout_ns);
+        // small batches: about one item per expert, fewer than the SMs can
+        // share evenly, so each item's columns are cut into 4 tasks
+        const int njt = (a.d + 255) / 256;
+        const int nsub = a.T <= kSmallDispatchMaxT ? std::min(4, njt) : 1;
+        const int grid6 = std::max(1, (int)std::min<long long>(sms, (long long)g.max_items * nsub));
+        down_gemm_kernel<<<grid6, kTcThreads, smem, st>>>(
+            mh, mwd, items, a.n_items, a.perm_token, a.d, njt, nsub, a.Y, g.ycap, a.yacc, a.overflow, a.status,
+            a.timeout_ns);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     combine_kernel<<<dim3(a.T, (a.d + 1023) / 1024), 128, 0, st>>>(a.bits, a.invpos, a.Y, g.ycap, a.yacc,
