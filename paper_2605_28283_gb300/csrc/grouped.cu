@@ -45,6 +45,8 @@ template <int NE>
 __global__ void __launch_bounds__(kTcThreads, 1)
     router_gemm_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant__ CUtensorMap map_wr,
                        int T, int E, int nk, int kpb, float* part, unsigned* status, uint64_t lim) {
+    pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
+    pdl_launch_dependents();
     constexpr int kStages = 4;
     constexpr int kTileB = NE * 128;
     constexpr int kStage = kTileBytesA + kTileB;
@@ -123,18 +125,33 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
 // ================================================================= selection
 // Selection from K-split partial logits (summed in split order).
+
+// Logit = sum over s of part[s * stride + off], added in split order; the
+// loads go out 8 at a time instead of one dependent round trip each.
+PP_DEVINL float sum_partials(const float* __restrict__ part, int nsplit, size_t stride, size_t off) {
+    float v = 0.0f;
+    int s = 0;
+    for (; s + 8 <= nsplit; s += 8) {
+        float q[8];
+#pragma unroll
+        for (int i = 0; i < 8; i++) q[i] = __ldg(part + (size_t)(s + i) * stride + off);
+#pragma unroll
+        for (int i = 0; i < 8; i++) v += q[i];
+    }
+    for (; s < nsplit; s++) v += __ldg(part + (size_t)s * stride + off);
+    return v;
+}
+
 template <int S>
 __global__ void __launch_bounds__(256) select_part_kernel(const float* __restrict__ part, int nsplit, int T, int E,
                                                           float p, int rule, int gate, int32_t* ids, int32_t* counts,
                                                           float* gates, float* logits_out, unsigned* status) {
+    pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
+    pdl_launch_dependents();
     const int lane = threadIdx.x & 31;
     const int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (t >= T) return;
-    auto load = [&](int j) {
-        float v = 0.0f;
-        for (int s = 0; s < nsplit; s++) v += part[((size_t)s * T + t) * E + j];
-        return v;
-    };
+    auto load = [&](int j) { return sum_partials(part, nsplit, (size_t)T * E, (size_t)t * E + j); };
     unsigned long long key[S];
     bool finite = true;
     const int k = warp_select<S>(load, E, p, rule, key, &finite);
@@ -156,13 +173,11 @@ __global__ void __launch_bounds__(256) select_part_cta_kernel(const float* __res
                                                               int E, float p, int rule, int gate, int32_t* ids,
                                                               int32_t* counts, float* gates, float* logits_out,
                                                               unsigned* status) {
+    pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
+    pdl_launch_dependents();
     __shared__ __align__(16) CtaSelScratch sc;
     const int t = blockIdx.x;
-    auto load = [&](int j) {
-        float v = 0.0f;
-        for (int s = 0; s < nsplit; s++) v += part[((size_t)s * T + t) * E + j];
-        return v;
-    };
+    auto load = [&](int j) { return sum_partials(part, nsplit, (size_t)T * E, (size_t)t * E + j); };
     bool on;
     int r;
     float g;
@@ -182,6 +197,8 @@ __global__ void __launch_bounds__(256) select_part_cta_kernel(const float* __res
 __global__ void dispatch_bits_kernel(const int32_t* __restrict__ ids, const int32_t* __restrict__ counts,
                                      const float* __restrict__ gates, int T, int E, uint32_t* bits, float* gexp,
                                      unsigned* status) {
+    pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
+    pdl_launch_dependents();
     const int t = blockIdx.x * blockDim.x + threadIdx.x;
     if (t >= T) return;
     uint32_t w[8] = {0, 0, 0, 0, 0, 0, 0, 0};
@@ -211,6 +228,8 @@ constexpr int kDispBlock = 256;
 
 __global__ void __launch_bounds__(kDispBlock) dispatch_count_kernel(const uint32_t* __restrict__ bits, int T, int E,
                                                                     int* wcnt, int* blkcnt) {
+    pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
+    pdl_launch_dependents();
     const int b = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int t = b * kDispBlock + threadIdx.x;
     uint32_t w[8];
@@ -238,6 +257,8 @@ __global__ void __launch_bounds__(kDispBlock) dispatch_count_kernel(const uint32
 __global__ void __launch_bounds__(kMaxExperts) dispatch_scan_kernel(const int* __restrict__ blkcnt, int nblk, int E,
                                                                     int* offsets, int* blkbase, WorkItem* items,
                                                                     int* n_items, int* overflow) {
+    pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
+    pdl_launch_dependents();
     const int e = threadIdx.x;
     if (e == 0) *overflow = 0;  // the down projection's overflow flag starts clear
     __shared__ int sh[kMaxExperts], si[kMaxExperts];
@@ -282,6 +303,8 @@ __global__ void __launch_bounds__(kDispBlock) dispatch_scatter_kernel(const uint
                                                                       const int* __restrict__ blkbase,
                                                                       int* perm_token, float* perm_gate,
                                                                       int* invpos) {
+    pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
+    pdl_launch_dependents();
     const int b = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int t = b * kDispBlock + threadIdx.x;
     const bool live = t < T;
@@ -319,6 +342,8 @@ __global__ void __launch_bounds__(1024) dispatch_small_kernel(const int32_t* __r
                                                               uint32_t* bits, int* offsets, WorkItem* items,
                                                               int* n_items, int* perm_token, float* perm_gate,
                                                               int* invpos, int* overflow, unsigned* status) {
+    pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
+    pdl_launch_dependents();
     __shared__ uint32_t mask[kMaxExperts][8];              // tokens of expert e
     __shared__ uint32_t dup[kSmallDispatchMaxT][8];        // entry (t, r) repeats an earlier id of token t
     __shared__ int off_s[kMaxExperts + 1], item_s[kMaxExperts + 1];
@@ -439,6 +464,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                    const int* __restrict__ n_items_p, const int* __restrict__ perm_token,
                    const float* __restrict__ perm_gate, int nk, int act, __nv_bfloat16* H, unsigned* status,
                    uint64_t lim) {
+    pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
+    pdl_launch_dependents();
     constexpr int kStages = NB == 128 ? 6 : 8;
     constexpr int kTileB = NB * 128;
     constexpr int kStage = kTileBytesA + kTileB;
@@ -583,6 +610,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                      const WorkItem* __restrict__ items, const int* __restrict__ n_items_p,
                      const int* __restrict__ perm_token, int d, int njt, int nsub, __nv_bfloat16* Y, long long ycap,
                      float* yacc, int* overflow, unsigned* status, uint64_t lim) {
+    pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
+    pdl_launch_dependents();
     constexpr int kStages = 4;
     constexpr int kTileB = 256 * 128;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -727,6 +756,8 @@ __global__ void __launch_bounds__(128) combine_kernel(const uint32_t* __restrict
                                                       const __nv_bfloat16* __restrict__ Y, long long ycap,
                                                       float* yacc, const int* __restrict__ overflow, int T, int E,
                                                       int d, __nv_bfloat16* y) {
+    pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
+    pdl_launch_dependents();
     const int t = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     __shared__ int pos_s[kMaxExperts];
     __shared__ int wn_s[4];
@@ -756,10 +787,19 @@ __global__ void __launch_bounds__(128) combine_kernel(const uint32_t* __restrict
         ya[0] = make_float4(0.f, 0.f, 0.f, 0.f);  // keep the accumulator zero at rest
         ya[1] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
-    for (int i = 0; i < n; i++) {
-        const uint4 v = *reinterpret_cast<const uint4*>(Y + (size_t)pos_s[i] * d + c);
-        acc[0] += bf16lo(v.x); acc[1] += bf16hi(v.x); acc[2] += bf16lo(v.y); acc[3] += bf16hi(v.y);
-        acc[4] += bf16lo(v.z); acc[5] += bf16hi(v.z); acc[6] += bf16lo(v.w); acc[7] += bf16hi(v.w);
+    // rows added in ascending expert order; their loads go out 4 at a time
+    for (int i0 = 0; i0 < n; i0 += 4) {
+        uint4 v4[4];
+#pragma unroll
+        for (int u = 0; u < 4; u++)
+            if (i0 + u < n) v4[u] = *reinterpret_cast<const uint4*>(Y + (size_t)pos_s[i0 + u] * d + c);
+#pragma unroll
+        for (int u = 0; u < 4; u++) {
+            if (i0 + u >= n) break;
+            const uint4 v = v4[u];
+            acc[0] += bf16lo(v.x); acc[1] += bf16hi(v.x); acc[2] += bf16lo(v.y); acc[3] += bf16hi(v.y);
+            acc[4] += bf16lo(v.z); acc[5] += bf16hi(v.z); acc[6] += bf16lo(v.w); acc[7] += bf16hi(v.w);
+        }
     }
     *reinterpret_cast<uint4*>(y + (size_t)t * d + c) =
         make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]), pack_bf16x2(acc[4], acc[5]),
@@ -768,6 +808,38 @@ __global__ void __launch_bounds__(128) combine_kernel(const uint32_t* __restrict
 
 // ====================================================================== host
 namespace {
+
+// Launch with programmatic dependent launch allowed: the kernel may be
+// scheduled while its predecessor on the stream finishes, and waits for it
+// in griddepcontrol.wait (pdl_wait) before touching memory.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args&&... args) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+    if (e == cudaErrorNotSupported) {
+        (void)cudaGetLastError();
+        cfg.numAttrs = 0;
+        e = cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+    }
+    return e;
+}
+
+// Launch through launch_pdl; returns the error from the enclosing function.
+#define PP_LAUNCH(...)                                   \
+    do {                                                 \
+        const cudaError_t le_ = launch_pdl(__VA_ARGS__); \
+        if (le_ != cudaSuccess) return le_;              \
+    } while (0)
+
 
 // bf16 [outer][inner] row-major, SW128 boxes.  `promote` is the L2 fill
 // granularity: 256 B where the neighbouring 128 B of a row is read next by
@@ -799,8 +871,8 @@ cudaError_t launch_router(const CUtensorMap& mx, const CUtensorMap& mwr, int T, 
     const size_t smem = 4 * (size_t)(kTileBytesA + NE * 128) + 1024;
     cudaError_t e = set_smem(router_gemm_kernel<NE>, smem);
     if (e != cudaSuccess) return e;
-    router_gemm_kernel<NE><<<dim3((T + 127) / 128, nsplit), kTcThreads, smem, st>>>(mx, mwr, T, E, nk, kpb, part,
-                                                                                     status, lim);
+    PP_LAUNCH(router_gemm_kernel<NE>, dim3((T + 127) / 128, nsplit), dim3(kTcThreads), smem, st, mx, mwr, T, E, nk,
+        kpb, part, status, lim);
     return cudaGetLastError();
 }
 
@@ -837,16 +909,20 @@ cudaError_t grouped_route(const GroupedArgs& a, cudaStream_t st) {
     }
     if (e != cudaSuccess) return e;
     if (a.T <= 64) {
-        select_part_cta_kernel<<<a.T, 256, 0, st>>>(a.part, g.nsplit, a.T, a.E, a.p, a.rule, a.gate, a.ids, a.counts,
-                                                    a.gates, a.logits_out, a.status);
+        PP_LAUNCH(select_part_cta_kernel, dim3(a.T), dim3(256), 0, st, a.part, g.nsplit, a.T, a.E, a.p, a.rule,
+            a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status);
         return cudaGetLastError();
     }
     const dim3 grid((a.T + 7) / 8), block(256);
     switch (sel_slots_for(a.E)) {
-        case 1: select_part_kernel<1><<<grid, block, 0, st>>>(a.part, g.nsplit, a.T, a.E, a.p, a.rule, a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status); break;
-        case 2: select_part_kernel<2><<<grid, block, 0, st>>>(a.part, g.nsplit, a.T, a.E, a.p, a.rule, a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status); break;
-        case 4: select_part_kernel<4><<<grid, block, 0, st>>>(a.part, g.nsplit, a.T, a.E, a.p, a.rule, a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status); break;
-        default: select_part_kernel<8><<<grid, block, 0, st>>>(a.part, g.nsplit, a.T, a.E, a.p, a.rule, a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status); break;
+        case 1: PP_LAUNCH(select_part_kernel<1>, dim3(grid), dim3(block), 0, st, a.part, g.nsplit, a.T, a.E, a.p, a.rule,
+                a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status); break;
+        case 2: PP_LAUNCH(select_part_kernel<2>, dim3(grid), dim3(block), 0, st, a.part, g.nsplit, a.T, a.E, a.p, a.rule,
+                a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status); break;
+        case 4: PP_LAUNCH(select_part_kernel<4>, dim3(grid), dim3(block), 0, st, a.part, g.nsplit, a.T, a.E, a.p, a.rule,
+                a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status); break;
+        default: PP_LAUNCH(select_part_kernel<8>, dim3(grid), dim3(block), 0, st, a.part, g.nsplit, a.T, a.E, a.p, a.rule,
+                a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status); break;
     }
     return cudaGetLastError();
 }
@@ -857,18 +933,18 @@ cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
     cudaError_t e;
     // dispatch
     if (a.T <= kSmallDispatchMaxT) {
-        dispatch_small_kernel<<<1, 1024, 0, st>>>(a.ids, a.counts, a.gates, a.T, a.E, a.bits, a.offsets,
-                                                  reinterpret_cast<WorkItem*>(a.items), a.n_items, a.perm_token,
-                                                  a.perm_gate, a.invpos, a.overflow, a.status);
+        PP_LAUNCH(dispatch_small_kernel, dim3(1), dim3(1024), 0, st, a.ids, a.counts, a.gates, a.T, a.E, a.bits,
+            a.offsets, reinterpret_cast<WorkItem*>(a.items), a.n_items, a.perm_token, a.perm_gate, a.invpos,
+            a.overflow, a.status);
     } else {
         const int nblk = (a.T + kDispBlock - 1) / kDispBlock;
-        dispatch_bits_kernel<<<(a.T + 255) / 256, 256, 0, st>>>(a.ids, a.counts, a.gates, a.T, a.E, a.bits,
-                                                                 a.gexp, a.status);
-        dispatch_count_kernel<<<nblk, kDispBlock, 0, st>>>(a.bits, a.T, a.E, a.wcnt, a.blkcnt);
-        dispatch_scan_kernel<<<1, kMaxExperts, 0, st>>>(a.blkcnt, nblk, a.E, a.offsets, a.blkbase,
-                                                       reinterpret_cast<WorkItem*>(a.items), a.n_items, a.overflow);
-        dispatch_scatter_kernel<<<nblk, kDispBlock, 0, st>>>(a.bits, a.gexp, a.T, a.E, a.wcnt, a.blkbase,
-                                                            a.perm_token, a.perm_gate, a.invpos);
+        PP_LAUNCH(dispatch_bits_kernel, dim3((a.T + 255) / 256), dim3(256), 0, st, a.ids, a.counts, a.gates, a.T, a.E,
+            a.bits, a.gexp, a.status);
+        PP_LAUNCH(dispatch_count_kernel, dim3(nblk), dim3(kDispBlock), 0, st, a.bits, a.T, a.E, a.wcnt, a.blkcnt);
+        PP_LAUNCH(dispatch_scan_kernel, dim3(1), dim3(kMaxExperts), 0, st, a.blkcnt, nblk, a.E, a.offsets, a.blkbase,
+            reinterpret_cast<WorkItem*>(a.items), a.n_items, a.overflow);
+        PP_LAUNCH(dispatch_scatter_kernel, dim3(nblk), dim3(kDispBlock), 0, st, a.bits, a.gexp, a.T, a.E, a.wcnt,
+            a.blkbase, a.perm_token, a.perm_gate, a.invpos);
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     // grouped gate/up
@@ -883,13 +959,13 @@ cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
     if (gated) {
         const size_t smem = 6 * (size_t)(kTileBytesA + 128 * 128) + 1024;
         if ((e = set_smem(gu_gemm_kernel<128>, smem)) != cudaSuccess) return e;
-        gu_gemm_kernel<128><<<grid, kTcThreads, smem, st>>>(mx1, mwg, mwu, items, a.n_items, a.perm_token, a.perm_gate,
-                                                            g.nk, a.act, a.H, a.status, a.timeout_ns);
+        PP_LAUNCH(gu_gemm_kernel<128>, dim3(grid), dim3(kTcThreads), smem, st, mx1, mwg, mwu, items, a.n_items,
+            a.perm_token, a.perm_gate, g.nk, a.act, a.H, a.status, a.timeout_ns);
     } else {
         const size_t smem = 8 * (size_t)(kTileBytesA + 64 * 128) + 1024;
         if ((e = set_smem(gu_gemm_kernel<64>, smem)) != cudaSuccess) return e;
-        gu_gemm_kernel<64><<<grid, kTcThreads, smem, st>>>(mx1, mwg, mwu, items, a.n_items, a.perm_token, a.perm_gate,
-                                                           g.nk, a.act, a.H, a.status, a.timeout_ns);
+        PP_LAUNCH(gu_gemm_kernel<64>, dim3(grid), dim3(kTcThreads), smem, st, mx1, mwg, mwu, items, a.n_items,
+            a.perm_token, a.perm_gate, g.nk, a.act, a.H, a.status, a.timeout_ns);
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     // grouped down + scatter-add
@@ -901,14 +977,12 @@ cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
         const int njt = (a.d + 255) / 256;
         const int nsub = a.T <= kSmallDispatchMaxT ? std::min(4, njt) : 1;
         const int grid6 = std::max(1, (int)std::min<long long>(sms, (long long)g.max_items * nsub));
-        down_gemm_kernel<<<grid6, kTcThreads, smem, st>>>(
-            mh, mwd, items, a.n_items, a.perm_token, a.d, njt, nsub, a.Y, g.ycap, a.yacc, a.overflow, a.status,
-            a.timeout_ns);
+        PP_LAUNCH(down_gemm_kernel, dim3(grid6), dim3(kTcThreads), smem, st, mh, mwd, items, a.n_items, a.perm_token,
+            a.d, njt, nsub, a.Y, g.ycap, a.yacc, a.overflow, a.status, a.timeout_ns);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
-    combine_kernel<<<dim3(a.T, (a.d + 1023) / 1024), 128, 0, st>>>(a.bits, a.invpos, a.Y, g.ycap, a.yacc,
-                                                                 a.overflow, a.T, a.E, a.d,
-                                                                 reinterpret_cast<__nv_bfloat16*>(a.y));
+    PP_LAUNCH(combine_kernel, dim3(a.T, (a.d + 1023) / 1024), dim3(128), 0, st, a.bits, a.invpos, a.Y, g.ycap,
+        a.yacc, a.overflow, a.T, a.E, a.d, reinterpret_cast<__nv_bfloat16*>(a.y));
     return cudaGetLastError();
 }
 
