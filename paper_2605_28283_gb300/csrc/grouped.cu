@@ -124,7 +124,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 }
 
 // ================================================================= selection
-// Selection from K-split partial logits (summed in split order).
+// Selection from K-split partial logits (summed in split order).  Up to
+// kCtaSelectMaxTokens tokens take one CTA each (the counting selection);
+// beyond, one warp per token (the warp sort).
+constexpr int kCtaSelectMaxTokens = 256;
 
 // Logit = sum over s of part[s * stride + off], added in split order; the
 // loads go out 8 at a time instead of one dependent round trip each.
@@ -194,32 +197,50 @@ __global__ void __launch_bounds__(256) select_part_cta_kernel(const float* __res
 // gexp[t][e]: the gate weight of that assignment (gates of a repeated id
 // add up), 0 where e is not activated.  Invalid ids and counts are recorded
 // and skipped.
-__global__ void dispatch_bits_kernel(const int32_t* __restrict__ ids, const int32_t* __restrict__ counts,
-                                     const float* __restrict__ gates, int T, int E, uint32_t* bits, float* gexp,
-                                     unsigned* status) {
+__global__ void __launch_bounds__(256) dispatch_bits_kernel(const int32_t* __restrict__ ids,
+                                                            const int32_t* __restrict__ counts,
+                                                            const float* __restrict__ gates, int T, int E,
+                                                            uint32_t* bits, float* gexp, unsigned* status) {
     pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
     pdl_launch_dependents();
-    const int t = blockIdx.x * blockDim.x + threadIdx.x;
+    // one warp per token: coalesced row writes
+    const int lane = threadIdx.x & 31;
+    const int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (t >= T) return;
-    uint32_t w[8] = {0, 0, 0, 0, 0, 0, 0, 0};
     float* grow = gexp + (size_t)t * E;
-    for (int e = 0; e < E; e++) grow[e] = 0.0f;
+    for (int e = lane; e < E; e += 32) grow[e] = 0.0f;
     int k = counts[t];
     if (k < 0 || k > E) {
-        record_status(status, PP_ERR_INVALID_ARG);
+        if (lane == 0) record_status(status, PP_ERR_INVALID_ARG);
         k = k < 0 ? 0 : E;
     }
-    for (int r = 0; r < k; r++) {
-        const int e = ids[(size_t)t * E + r];
-        if (e < 0 || e >= E) {
+    __syncwarp();
+    uint32_t w[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    // entries in rank order, one lane each; repeated ids add their gates in
+    // rank order (the lanes of a round take turns on a repeated id)
+    for (int r0 = 0; r0 < k; r0 += 32) {
+        const int r = r0 + lane;
+        int e = r < k ? ids[(size_t)t * E + r] : -1;
+        if (r < k && (e < 0 || e >= E)) {
             record_status(status, PP_ERR_INVALID_ARG);
-            continue;
+            e = -1;
         }
-        w[e >> 5] |= 1u << (e & 31);
-        grow[e] += gates[(size_t)t * E + r];
+        const float gv = e >= 0 ? gates[(size_t)t * E + r] : 0.0f;
+        if (e >= 0) w[e >> 5] |= 1u << (e & 31);
+        for (int l = 0; l < 32; l++) {
+            const int el = __shfl_sync(kFull, e, l);
+            const float gl = __shfl_sync(kFull, gv, l);
+            if (el >= 0 && lane == (el & 31)) grow[el] += gl;
+            __syncwarp();
+        }
     }
 #pragma unroll
-    for (int i = 0; i < 8; i++) bits[(size_t)t * 8 + i] = w[i];
+    for (int i = 0; i < 8; i++) {
+        uint32_t v = w[i];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) v |= __shfl_xor_sync(kFull, v, o);
+        if (lane == i) bits[(size_t)t * 8 + i] = v;
+    }
 }
 
 // Token block b (256 tokens, one per thread): per-warp counts of every
@@ -308,6 +329,13 @@ __global__ void __launch_bounds__(kDispBlock) dispatch_scatter_kernel(const uint
     const int b = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int t = b * kDispBlock + threadIdx.x;
     const bool live = t < T;
+    // this block's bases, per warp: blkbase[b][e] + wcnt[b][warp][e]
+    __shared__ int base_s[8][kMaxExperts];
+    for (int i = threadIdx.x; i < 8 * E; i += kDispBlock) {
+        const int v = i / E, e = i - v * E;
+        base_s[v][e] = blkbase[(size_t)b * E + e] + wcnt[((size_t)b * 8 + v) * E + e];
+    }
+    __syncthreads();
     uint32_t w[8];
 #pragma unroll
     for (int i = 0; i < 8; i++) w[i] = live ? bits[(size_t)t * 8 + i] : 0u;
@@ -316,7 +344,7 @@ __global__ void __launch_bounds__(kDispBlock) dispatch_scatter_kernel(const uint
         const bool on = (w[e >> 5] >> (e & 31)) & 1u;
         const unsigned bal = __ballot_sync(kFull, on);
         if (on) {
-            const int pos = blkbase[(size_t)b * E + e] + wcnt[((size_t)b * 8 + warp) * E + e] + __popc(bal & lt);
+            const int pos = base_s[warp][e] + __popc(bal & lt);
             perm_token[pos] = t;
             perm_gate[pos] = gexp[(size_t)t * E + e];
             invpos[(size_t)t * E + e] = pos;
@@ -908,7 +936,7 @@ cudaError_t grouped_route(const GroupedArgs& a, cudaStream_t st) {
         default: e = launch_router<256>(mx, mwr, a.T, a.E, g.nk, g.kpb, g.nsplit, a.part, a.status, a.timeout_ns, st); break;
     }
     if (e != cudaSuccess) return e;
-    if (a.T <= 64) {
+    if (a.T <= kCtaSelectMaxTokens) {
         PP_LAUNCH(select_part_cta_kernel, dim3(a.T), dim3(256), 0, st, a.part, g.nsplit, a.T, a.E, a.p, a.rule,
             a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status);
         return cudaGetLastError();
@@ -938,7 +966,7 @@ cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
             a.overflow, a.status);
     } else {
         const int nblk = (a.T + kDispBlock - 1) / kDispBlock;
-        PP_LAUNCH(dispatch_bits_kernel, dim3((a.T + 255) / 256), dim3(256), 0, st, a.ids, a.counts, a.gates, a.T, a.E,
+        PP_LAUNCH(dispatch_bits_kernel, dim3((a.T + 7) / 8), dim3(256), 0, st, a.ids, a.counts, a.gates, a.T, a.E,
             a.bits, a.gexp, a.status);
         PP_LAUNCH(dispatch_count_kernel, dim3(nblk), dim3(kDispBlock), 0, st, a.bits, a.T, a.E, a.wcnt, a.blkcnt);
         PP_LAUNCH(dispatch_scan_kernel, dim3(1), dim3(kMaxExperts), 0, st, a.blkcnt, nblk, a.E, a.offsets, a.blkbase,
