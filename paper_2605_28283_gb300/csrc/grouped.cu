@@ -357,7 +357,8 @@ __global__ void __launch_bounds__(kDispBlock) dispatch_scatter_kernel(const uint
 // experts cost more than their work).  Shared memory holds, per expert, the
 // 256-bit mask of the tokens that activated it; an assignment (t, e) lands
 // at offsets[e] + (tokens below t in e's mask), so tokens stay in ascending
-// order within each expert, as in the multi-block path.  Writes the same
+// order within each expert, as in the multi-block path; work items hold at
+// most item_rows rows.  Writes the same
 // outputs as that path (bits, offsets, work items, perm_token, perm_gate,
 // invpos) and clears the overflow flag of the down projection.  Gates of a
 // repeated id add up (with three or more copies the order of the additions
@@ -369,7 +370,8 @@ __global__ void __launch_bounds__(1024) dispatch_small_kernel(const int32_t* __r
                                                               const float* __restrict__ gates, int T, int E,
                                                               uint32_t* bits, int* offsets, WorkItem* items,
                                                               int* n_items, int* perm_token, float* perm_gate,
-                                                              int* invpos, int* overflow, unsigned* status) {
+                                                              int* invpos, int* overflow, int item_rows,
+                                                              unsigned* status) {
     pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
     pdl_launch_dependents();
     __shared__ uint32_t mask[kMaxExperts][8];              // tokens of expert e
@@ -411,7 +413,7 @@ __global__ void __launch_bounds__(1024) dispatch_small_kernel(const int32_t* __r
 #pragma unroll
                 for (int w = 0; w < 8; w++) n += __popc(mask[e][w]);
             c[q] = n;
-            m[q] = (n + 127) >> 7;
+            m[q] = (n + item_rows - 1) / item_rows;
             cs += n;
             ms += m[q];
         }
@@ -442,7 +444,7 @@ __global__ void __launch_bounds__(1024) dispatch_small_kernel(const int32_t* __r
         const int e = tid, o = off_s[e], n = off_s[e + 1] - o;
         offsets[e] = o;
         int it = item_s[e];
-        for (int a0 = 0; a0 < n; a0 += 128) items[it++] = WorkItem{e, o + a0, min(128, n - a0), 0};
+        for (int a0 = 0; a0 < n; a0 += item_rows) items[it++] = WorkItem{e, o + a0, min(item_rows, n - a0), 0};
     }
     if (tid == 0) {
         offsets[E] = off_s[kMaxExperts];
@@ -774,6 +776,287 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (warp == 1) tmem_dealloc(tmem, 512);
 }
 
+// ========================================================== small batches
+// Operand-swapped grouped GEMMs for items of at most kSwN tokens (batches of
+// up to kSwapMaxT tokens, where an expert sees a few tokens): the weights are the
+// M = 128 operand and the item's tokens the N = kSwN operand.  A pipeline
+// stage is then 16 KB of weights + 2 KB of token rows (a 128-token tile would
+// spend half of every stage on padding rows), so about twice as many weight
+// bytes are in flight per SM.
+constexpr int kSwN = 16;
+constexpr int kSwapMaxT = 128;  // batches above this keep 128-row items (experts see more tokens)
+constexpr int kSwTileW = 128 * 128;   // 128 weight rows x 64 bf16
+constexpr int kSwTileX = kSwN * 128;  // kSwN token rows x 64 bf16
+
+// Gate/up (SwiGLU): D[128 x kSwN] = [64 gate rows; 64 up rows of expert e]
+// . x_tokens^T over K = d.  TMEM lanes 0-63 hold the gate sums of neurons
+// 0-63, lanes 64-127 the up sums; the warps reading the up lanes hand them to
+// the gate warps through shared memory, which write h = silu(g) * u * gate.
+__global__ void __launch_bounds__(kTcThreads, 1)
+    gu_swap_kernel(const __grid_constant__ CUtensorMap map_x1, const __grid_constant__ CUtensorMap map_wg,
+                   const __grid_constant__ CUtensorMap map_wu, const WorkItem* __restrict__ items,
+                   const int* __restrict__ n_items_p, const int* __restrict__ perm_token,
+                   const float* __restrict__ perm_gate, int nk, __nv_bfloat16* H, unsigned* status, uint64_t lim) {
+    pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
+    pdl_launch_dependents();
+    constexpr int kStages = 11;
+    constexpr int kStage = kSwTileW + kSwTileX;  // 18 KB, a multiple of 1024
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    __shared__ uint64_t full[kStages], empty[kStages], tfull[2], tempty[2];
+    __shared__ uint32_t taddr_s;
+    __shared__ float up_s[2][32][kSwN + 1];  // up sums of neurons 0-31 / 32-63 for the gate warps
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n_items = *n_items_p;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kStages; i++) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        for (int i = 0; i < 2; i++) {
+            mbar_init(&tfull[i], 1);
+            mbar_init(&tempty[i], 4);
+        }
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(&taddr_s, 32);  // two kSwN-column accumulators
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = taddr_s;
+
+    if (warp == 0) {
+        int it = 0;
+        // the next item and its token rows are read one item ahead
+        WorkItem wn = blockIdx.x < n_items ? items[blockIdx.x] : WorkItem{0, 0, 1, 0};
+        int tokn = blockIdx.x < n_items ? perm_token[wn.a0 + min(lane & (kSwN - 1), wn.cnt - 1)] : 0;
+        for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x) {
+            const WorkItem w = wn;
+            // lane i < kSwN: the item's i-th token row (padding repeats the last)
+            const int tok = tokn;
+            if (wi + (int)gridDim.x < n_items) {
+                wn = items[wi + gridDim.x];
+                tokn = perm_token[wn.a0 + min(lane & (kSwN - 1), wn.cnt - 1)];
+            }
+            const int ng = (w.cnt + 3) >> 2;  // gather4 groups of live rows
+            const int r0 = __shfl_sync(kFull, tok, (4 * lane) & 31), r1 = __shfl_sync(kFull, tok, (4 * lane + 1) & 31);
+            const int r2 = __shfl_sync(kFull, tok, (4 * lane + 2) & 31), r3 = __shfl_sync(kFull, tok, (4 * lane + 3) & 31);
+            for (int kc = 0; kc < nk; kc++, it++) {
+                const int s = it % kStages;
+                unsigned char* st = smem + (size_t)s * kStage;
+                if (lane == 0) {
+                    if (it >= kStages) mbar_wait(&empty[s], (uint32_t)((it / kStages) - 1) & 1u, status, lim);
+                    mbar_arrive_expect_tx(&full[s], (uint32_t)(kSwTileW + ng * 512));
+                }
+                __syncwarp();
+                if (lane < ng) tma_gather4(st + kSwTileW + lane * 512, &map_x1, kc * 64, r0, r1, r2, r3, &full[s]);
+                if (lane == 0) {
+                    tma_load_2d(st, &map_wg, kc * 64, w.e * 64, &full[s]);
+                    tma_load_2d(st + 64 * 128, &map_wu, kc * 64, w.e * 64, &full[s]);
+                }
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16_m128(kSwN);
+            int it = 0, acc = 0;
+            for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x, acc++) {
+                const int a = acc & 1;
+                if (acc >= 2) mbar_wait(&tempty[a], (uint32_t)((acc >> 1) - 1) & 1u, status, lim);
+                tc_fence_after();
+                for (int kc = 0; kc < nk; kc++, it++) {
+                    const int s = it % kStages;
+                    mbar_wait(&full[s], (uint32_t)(it / kStages) & 1u, status, lim);
+                    tc_fence_after();
+                    unsigned char* st = smem + (size_t)s * kStage;
+                    umma_k64(tmem + (uint32_t)(a * kSwN), st, st + kSwTileW, idesc, kc > 0);
+                    umma_commit(&empty[s]);
+                }
+                umma_commit(&tfull[a]);
+            }
+        }
+        __syncwarp();
+    } else {
+        const int q = warp & 3;  // TMEM lanes 32 q .. 32 q + 31
+        int acc = 0;
+        for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x, acc++) {
+            const WorkItem w = items[wi];
+            const int a = acc & 1;
+            const float gw_l = lane < w.cnt ? perm_gate[w.a0 + lane] : 0.0f;  // gate weight of token `lane`
+            mbar_wait(&tfull[a], (uint32_t)(acc >> 1) & 1u, status, lim);
+            tc_fence_after();
+            uint32_t v[kSwN];
+            tmem_ld16(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(a * kSwN), v);
+            tmem_ld_wait();
+            if (q >= 2) {
+#pragma unroll
+                for (int t = 0; t < kSwN; t++) up_s[q - 2][lane][t] = __uint_as_float(v[t]);
+            }
+            named_bar_sync(1, 128);
+            if (q < 2) {
+                const int n = 32 * q + lane;  // this lane's neuron
+#pragma unroll
+                for (int t = 0; t < kSwN; t++) {
+                    const float gw = __shfl_sync(kFull, gw_l, t);
+                    if (t < w.cnt) {
+                        const float h = act_h(PP_ACT_SWIGLU, up_s[q][lane][t], __uint_as_float(v[t])) * gw;
+                        H[(size_t)(w.a0 + t) * 64 + n] = __float2bfloat16_rn(h);
+                    }
+                }
+            }
+            named_bar_sync(1, 128);  // up_s is free for the next item
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[a]);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) tmem_dealloc(tmem, 32);
+}
+
+// Down projection: per task (item, part of the ceil(d / 128) row tiles),
+// D[128 x kSwN] = W_down[128 rows, 64 columns of expert e] . H_item^T; the
+// item's kSwN H rows stay in shared memory for the task while the W_down
+// tiles stream through the ring (two H buffers, so that the next task's
+// tiles follow without a gap).  Lane = output row, column t = token: Y row
+// a0 + t (or, past ycap, a reduction into yacc) receives it.
+__global__ void __launch_bounds__(kTcThreads, 1)
+    down_swap_kernel(const __grid_constant__ CUtensorMap map_h, const __grid_constant__ CUtensorMap map_wd,
+                     const WorkItem* __restrict__ items, const int* __restrict__ n_items_p,
+                     const int* __restrict__ perm_token, int d, int nrt, int nsub, __nv_bfloat16* Y, long long ycap,
+                     float* yacc, int* overflow, unsigned* status, uint64_t lim) {
+    pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
+    pdl_launch_dependents();
+    constexpr int kStages = 12;
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    unsigned char* tileH = smem;                // 2 x kSwTileX bytes (1024-aligned)
+    unsigned char* ring = smem + 2 * 2048;      // kStages x kSwTileW
+    __shared__ uint64_t full[kStages], empty[kStages], tfull[2], tempty[2], hfull[2], hempty[2];
+    __shared__ uint32_t taddr_s;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n_tasks = *n_items_p * nsub;
+    auto tiles = [&](int v, int& r0, int& r1) {  // row tiles [r0, r1) of task v
+        const int sp = v % nsub;
+        r0 = sp * nrt / nsub;
+        r1 = (sp + 1) * nrt / nsub;
+    };
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kStages; i++) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        for (int i = 0; i < 2; i++) {
+            mbar_init(&tfull[i], 1);
+            mbar_init(&tempty[i], 4);
+        }
+        for (int i = 0; i < 2; i++) {
+            mbar_init(&hfull[i], 1);
+            mbar_init(&hempty[i], 1);
+        }
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(&taddr_s, 32);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = taddr_s;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int it = 0, ii = 0;
+            WorkItem wn = blockIdx.x < n_tasks ? items[blockIdx.x / nsub] : WorkItem{0, 0, 0, 0};
+            for (int v = blockIdx.x; v < n_tasks; v += gridDim.x, ii++) {
+                const WorkItem w = wn;
+                if (v + (int)gridDim.x < n_tasks) wn = items[(v + gridDim.x) / nsub];  // next task's item, early
+                int r0, r1;
+                tiles(v, r0, r1);
+                const int hb = ii & 1;
+                if (ii >= 2) mbar_wait(&hempty[hb], (uint32_t)((ii >> 1) - 1) & 1u, status, lim);
+                mbar_arrive_expect_tx(&hfull[hb], kSwTileX);
+                tma_load_2d(tileH + hb * 2048, &map_h, 0, w.a0, &hfull[hb]);
+                for (int rt = r0; rt < r1; rt++, it++) {
+                    const int s = it % kStages;
+                    if (it >= kStages) mbar_wait(&empty[s], (uint32_t)((it / kStages) - 1) & 1u, status, lim);
+                    mbar_arrive_expect_tx(&full[s], kSwTileW);
+                    tma_load_2d(ring + (size_t)s * kSwTileW, &map_wd, w.e * 64, rt * 128, &full[s]);
+                }
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16_m128(kSwN);
+            int it = 0, acc = 0, ii = 0;
+            for (int v = blockIdx.x; v < n_tasks; v += gridDim.x, ii++) {
+                int r0, r1;
+                tiles(v, r0, r1);
+                const int hb = ii & 1;
+                mbar_wait(&hfull[hb], (uint32_t)(ii >> 1) & 1u, status, lim);
+                for (int rt = r0; rt < r1; rt++, it++, acc++) {
+                    const int a = acc & 1;
+                    if (acc >= 2) mbar_wait(&tempty[a], (uint32_t)((acc >> 1) - 1) & 1u, status, lim);
+                    const int s = it % kStages;
+                    mbar_wait(&full[s], (uint32_t)(it / kStages) & 1u, status, lim);
+                    tc_fence_after();
+                    umma_k64(tmem + (uint32_t)(a * kSwN), ring + (size_t)s * kSwTileW, tileH + hb * 2048, idesc,
+                             false);
+                    umma_commit(&empty[s]);
+                    umma_commit(&tfull[a]);
+                }
+                umma_commit(&hempty[hb]);
+            }
+        }
+        __syncwarp();
+    } else {
+        const int q = warp & 3;
+        int acc = 0;
+        for (int v = blockIdx.x; v < n_tasks; v += gridDim.x) {
+            const WorkItem w = items[v / nsub];
+            int r0, r1;
+            tiles(v, r0, r1);
+            // token of assignment row a0 + lane (for rows past ycap)
+            const long long arow_l = (long long)w.a0 + lane;
+            const int tok_l = lane < w.cnt && arow_l >= ycap ? perm_token[arow_l] : -1;
+            if (lane == 0 && (long long)w.a0 + w.cnt > ycap) *overflow = 1;
+            for (int rt = r0; rt < r1; rt++, acc++) {
+                const int a = acc & 1;
+                mbar_wait(&tfull[a], (uint32_t)(acc >> 1) & 1u, status, lim);
+                tc_fence_after();
+                uint32_t val[kSwN];
+                tmem_ld16(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(a * kSwN), val);
+                tmem_ld_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&tempty[a]);
+                const int row = rt * 128 + 32 * q + lane;  // output element of d
+#pragma unroll
+                for (int t = 0; t < kSwN; t++) {
+                    const int tk = __shfl_sync(kFull, tok_l, t);
+                    if (t < w.cnt && row < d) {
+                        const long long arow = (long long)w.a0 + t;
+                        if (arow < ycap)
+                            Y[(size_t)arow * d + row] = __float2bfloat16_rn(__uint_as_float(val[t]));
+                        else
+                            atomicAdd(&yacc[(size_t)tk * d + row], __uint_as_float(val[t]));
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) tmem_dealloc(tmem, 32);
+}
+
 // =================================================================== combine
 // y[t] = the sum of token t's assignment rows Y[pos] in ascending expert
 // order, plus yacc[t] when the down projection overflowed (yacc is then
@@ -914,7 +1197,8 @@ GroupedPlan grouped_plan(int T, int d, int E, int sms) {
     const int ns = std::max(1, std::min(sms / mt, std::min(g.nk / 4, 64)));
     g.kpb = (g.nk + ns - 1) / ns;
     g.nsplit = (g.nk + g.kpb - 1) / g.kpb;
-    g.max_items = (int)std::min<long long>((long long)T * E / 128 + E + 1, (long long)T * E);
+    const int rows = T <= kSwapMaxT ? kSwN : 128;  // rows per work item
+    g.max_items = (int)std::min<long long>((long long)T * E / rows + E + 1, (long long)T * E);
     g.nnz_max = (long long)T * E;
     g.ycap = (long long)T * std::min(E, 64);  // assignment rows kept for the combine
     return g;
@@ -963,7 +1247,7 @@ cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
     if (a.T <= kSmallDispatchMaxT) {
         PP_LAUNCH(dispatch_small_kernel, dim3(1), dim3(1024), 0, st, a.ids, a.counts, a.gates, a.T, a.E, a.bits,
             a.offsets, reinterpret_cast<WorkItem*>(a.items), a.n_items, a.perm_token, a.perm_gate, a.invpos,
-            a.overflow, a.status);
+            a.overflow, a.T <= kSwapMaxT ? kSwN : 128, a.status);
     } else {
         const int nblk = (a.T + kDispBlock - 1) / kDispBlock;
         PP_LAUNCH(dispatch_bits_kernel, dim3((a.T + 7) / 8), dim3(256), 0, st, a.ids, a.counts, a.gates, a.T, a.E,
@@ -984,7 +1268,15 @@ cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
         return cudaErrorInvalidValue;
     const int grid = std::max(1, std::min(sms, g.max_items));
     const WorkItem* items = reinterpret_cast<const WorkItem*>(a.items);
-    if (gated) {
+    // batches of up to kSwapMaxT tokens: items of at most kSwN rows and the
+    // operand-swapped kernels (weights as the M = 128 operand)
+    const bool small = a.T <= kSwapMaxT;
+    if (gated && small) {
+        const size_t smem = 11 * (size_t)(kSwTileW + kSwTileX) + 1024;
+        if ((e = set_smem(gu_swap_kernel, smem)) != cudaSuccess) return e;
+        PP_LAUNCH(gu_swap_kernel, dim3(grid), dim3(kTcThreads), smem, st, mx1, mwg, mwu, items, a.n_items,
+            a.perm_token, a.perm_gate, g.nk, a.H, a.status, a.timeout_ns);
+    } else if (gated) {
         const size_t smem = 6 * (size_t)(kTileBytesA + 128 * 128) + 1024;
         if ((e = set_smem(gu_gemm_kernel<128>, smem)) != cudaSuccess) return e;
         PP_LAUNCH(gu_gemm_kernel<128>, dim3(grid), dim3(kTcThreads), smem, st, mx1, mwg, mwu, items, a.n_items,
@@ -997,11 +1289,26 @@ cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     // grouped down + scatter-add
-    {
+    if (small) {
+        CUtensorMap mh16, mwd128;
+        if (!encode_2d(&mh16, a.H, 64, (uint64_t)g.nnz_max + 128, 64, kSwN) ||
+            !encode_2d(&mwd128, a.Wd, (uint64_t)a.E * 64, a.d, 64, 128, CU_TENSOR_MAP_L2_PROMOTION_L2_128B))
+            return cudaErrorInvalidValue;
+        const size_t smem = 2 * 2048 + 12 * (size_t)kSwTileW + 1024;
+        if ((e = set_smem(down_swap_kernel, smem)) != cudaSuccess) return e;
+        // each item's ceil(d / 128) row tiles cut into up to 4 tasks, so that
+        // every SM streams W_down
+        const int nrt = (a.d + 127) / 128;
+        const int nsub = std::min(4, nrt);
+        const int grid6 = std::max(1, (int)std::min<long long>(sms, (long long)g.max_items * nsub));
+        PP_LAUNCH(down_swap_kernel, dim3(grid6), dim3(kTcThreads), smem, st, mh16, mwd128, items, a.n_items,
+            a.perm_token, a.d, nrt, nsub, a.Y, g.ycap, a.yacc, a.overflow, a.status, a.timeout_ns);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    } else {
         const size_t smem = (size_t)kTileBytesA + 4 * (size_t)256 * 128 + 1024;
         if ((e = set_smem(down_gemm_kernel, smem)) != cudaSuccess) return e;
-        // small batches: about one item per expert, fewer than the SMs can
-        // share evenly, so each item's columns are cut into 4 tasks
+        // up to 256 tokens: about one 128-row item per expert, fewer than the
+        // SMs can share evenly, so each item's columns are cut into 4 tasks
         const int njt = (a.d + 255) / 256;
         const int nsub = a.T <= kSmallDispatchMaxT ? std::min(4, njt) : 1;
         const int grid6 = std::max(1, (int)std::min<long long>(sms, (long long)g.max_items * nsub));
