@@ -214,24 +214,32 @@ def layer_flops(w, B, k_sum):
     return 2.0 * B * w.n_experts * w.d_model + 2.0 * k_sum * mats * 64 * w.d_model
 
 
-def kernel_traffic(workload, p, B):
+def kernel_traffic(workload, p, B, kind="decode"):
     """DRAM bytes per layer call measured by ncu (committed summary), valid
-    only while the kernel sources are unchanged; None otherwise."""
+    only while the kernel's sources are unchanged; None otherwise."""
     path = os.path.join(ROOT, "profiles", "dram_traffic.json")
     try:
         rec = json.load(open(path))
     except Exception:
         return None
-    if rec.get("sources_sha") != sources_sha():
-        return None
     ent = rec.get("entries", {}).get("%s@p%g@B%d" % (workload, p, B))
-    return None if ent is None else ent.get("dram_bytes_per_layer")
+    if ent is None or ent.get("sources_sha") != sources_sha(kind):
+        return None
+    return ent.get("dram_bytes_per_layer")
 
 
-def sources_sha():
+# source files each timed kernel is built from: a DRAM-traffic record stays
+# valid while these are unchanged
+KERNEL_SOURCES = {
+    "decode": ["decode.cu", "pp_common.cuh", "pp_select.cuh", "pp_kernels.h", "api.cu"],
+    "grouped": ["grouped.cu", "pp_common.cuh", "pp_select.cuh", "pp_tc.cuh", "pp_kernels.h", "api.cu"],
+}
+
+
+def sources_sha(kind="decode"):
     h = hashlib.sha256()
     d = os.path.join(ROOT, "paper_2605_28283_gb300", "csrc")
-    for n in sorted(os.listdir(d)):
+    for n in sorted(KERNEL_SOURCES[kind]):
         with open(os.path.join(d, n), "rb") as f:
             h.update(n.encode() + f.read())
     return h.hexdigest()[:16]
@@ -428,7 +436,7 @@ def main():
                               "launch_ms": per_launch_ms, "bytes_per_launch": bytes_per_launch,
                               "flops_per_launch": flops_per_launch, "roofline_bound": roof["bound"],
                               "achieved": achieved, "peak": peak, "frac": achieved / peak,
-                              "sources_sha": sources_sha()}))
+                              "sources_sha": sources_sha("decode" if B <= 4 or w.dtype == "f32" else "grouped")}))
         return
 
     # ---- warm-L2 number (no flush), for context
@@ -495,7 +503,8 @@ def main():
                       "l2": "no flush (warm)" if args.no_flush else "flushed between steps (256 MiB write, untimed)",
                       "parallelism": "replicas" if world > 1 else "single GPU"},
            "roofline": dict(roof, achieved=achieved, peak=peak, frac=achieved / peak,
-                            traffic=kernel_traffic(w.name, args.p, B), peak_kind=peak_kind,
+                            traffic=kernel_traffic(w.name, args.p, B, "decode" if B <= 4 or w.dtype == "f32" else "grouped"),
+                            peak_kind=peak_kind,
                             kernel="decode_layer_kernel" if B <= 4 else "pp_layer (grouped tcgen05 path)",
                             per="one pp_layer call (one layer)", launch_ms=per_launch_ms),
            "expert_bytes": {"gbs": expert_gbs, "frac_of_peak": expert_gbs / hbm_peak,

@@ -329,10 +329,12 @@ __global__ void __launch_bounds__(kDispBlock) dispatch_scatter_kernel(const uint
     const int b = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int t = b * kDispBlock + threadIdx.x;
     const bool live = t < T;
+    // experts [e0, e1) of this block (blockIdx.y splits the expert loop)
+    const int e0 = blockIdx.y * E / gridDim.y, e1 = (blockIdx.y + 1) * E / gridDim.y;
     // this block's bases, per warp: blkbase[b][e] + wcnt[b][warp][e]
     __shared__ int base_s[8][kMaxExperts];
-    for (int i = threadIdx.x; i < 8 * E; i += kDispBlock) {
-        const int v = i / E, e = i - v * E;
+    for (int i = threadIdx.x; i < 8 * (e1 - e0); i += kDispBlock) {
+        const int v = i / (e1 - e0), e = e0 + i - v * (e1 - e0);
         base_s[v][e] = blkbase[(size_t)b * E + e] + wcnt[((size_t)b * 8 + v) * E + e];
     }
     __syncthreads();
@@ -340,7 +342,7 @@ __global__ void __launch_bounds__(kDispBlock) dispatch_scatter_kernel(const uint
 #pragma unroll
     for (int i = 0; i < 8; i++) w[i] = live ? bits[(size_t)t * 8 + i] : 0u;
     const unsigned lt = (1u << lane) - 1u;
-    for (int e = 0; e < E; e++) {
+    for (int e = e0; e < e1; e++) {
         const bool on = (w[e >> 5] >> (e & 31)) & 1u;
         const unsigned bal = __ballot_sync(kFull, on);
         if (on) {
@@ -1255,7 +1257,7 @@ cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
         PP_LAUNCH(dispatch_count_kernel, dim3(nblk), dim3(kDispBlock), 0, st, a.bits, a.T, a.E, a.wcnt, a.blkcnt);
         PP_LAUNCH(dispatch_scan_kernel, dim3(1), dim3(kMaxExperts), 0, st, a.blkcnt, nblk, a.E, a.offsets, a.blkbase,
             reinterpret_cast<WorkItem*>(a.items), a.n_items, a.overflow);
-        PP_LAUNCH(dispatch_scatter_kernel, dim3(nblk), dim3(kDispBlock), 0, st, a.bits, a.gexp, a.T, a.E, a.wcnt,
+        PP_LAUNCH(dispatch_scatter_kernel, dim3(nblk, std::min(8, a.E)), dim3(kDispBlock), 0, st, a.bits, a.gexp, a.T, a.E, a.wcnt,
             a.blkbase, a.perm_token, a.perm_gate, a.invpos);
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
