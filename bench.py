@@ -60,6 +60,24 @@ def dist_env():
     return rank, world, local
 
 
+def max_over_ranks(v, world, device):
+    """The largest of the ranks' values (every rank gets it); v itself for one rank."""
+    if world == 1:
+        return v
+    import torch
+    t = torch.tensor([v], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_throughput(units_per_rank, seconds, world, device):
+    """Whole-job throughput of `world` independent replicas that each
+    processed units_per_rank units: all units over the slowest rank's time.
+    Returns (units/s, slowest time)."""
+    slowest = max_over_ranks(seconds, world, device)
+    return world * units_per_rank / slowest, slowest
+
+
 def load_peaks():
     """(HBM GB/s, dense bf16 TFLOP/s sustained, kind): measured copy and GEMM
     figures for this GPU pool, else the recipe's fallback numbers."""
@@ -297,7 +315,8 @@ def run_reference(args):
     el = time.perf_counter() - t0
     per_step_model = el / steps * w.n_layers
     value = args.batch / per_step_model
-    cores = 1
+    # the oracle's OpenMP loops run over tokens
+    cores = max(1, min(int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1)), args.batch))
     out = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus, "steps": steps,
            "warmup": args.warmup, "ms_per_step": per_step_model * 1e3, "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
@@ -348,13 +367,6 @@ def main():
             torch.distributed.barrier()
         torch.cuda.synchronize()
 
-    def max_over_ranks(v):
-        if world == 1:
-            return v
-        t = torch.tensor([v], dtype=torch.float64, device=device)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        return float(t.item())
-
     # ---- headline: p = args.p
     pf = float(np.float32(args.p))
     graphs = capture_graphs(pp, desc, layers, pf, B, args.pool, ws, stream)
@@ -364,12 +376,12 @@ def main():
     times = time_graphs(graphs, args.steps, args.warmup, flush, stream, profile_range=True)
     barrier()
     clocks = sampler.stop()
-    total_ms = max_over_ranks(sum(times))
+    value, slowest_s = replica_throughput(B * args.steps, sum(times) / 1e3, world, device)
+    total_ms = slowest_s * 1e3
     status = pp.pp_get_device_status(ws)
     if status != pp.PP_OK:
         raise SystemExit("device status: %s" % pp.status_name(status))
     ms_per_step = total_ms / args.steps
-    value = world * B * args.steps / (total_ms / 1e3)
 
     # bytes per step from the actual selections of the pool entries
     ks, union = selection_stats(pp, desc, layers, w, pf, B, args.pool, ws)
@@ -484,14 +496,13 @@ def main():
                     y_host.copy_(y_dev, non_blocking=True)
                     stream.synchronize()
                 timings[mode] = time.perf_counter() - t0
-    el_max = max_over_ranks(timings["graph"])
-    e2e = {"value": world * B * e2e_steps / el_max,
+    e2e = {"value": replica_throughput(B * e2e_steps, timings["graph"], world, device)[0],
            "unit": "tokens/s", "h2d_bytes_per_step": w.n_layers * B * w.d_model * esz,
            "d2h_bytes_per_step": w.n_layers * B * w.d_model * esz,
            "path": "pp_layer via the ctypes binding, 32 calls captured once in a CUDA graph; per step one "
                    "pinned H2D copy of the 32 layer inputs, graph replay, one D2H copy of the 32 outputs, "
                    "host synchronisation",
-           "eager_value": world * B * e2e_steps / max_over_ranks(timings["eager"]),
+           "eager_value": replica_throughput(B * e2e_steps, timings["eager"], world, device)[0],
            "eager_path": "the same with the 32 pp_layer calls made eagerly every step"}
 
     out = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
