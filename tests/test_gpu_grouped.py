@@ -15,7 +15,7 @@ pytestmark = pytest.mark.gpu
 
 
 @pytest.mark.parametrize("T,p", [(5, 0.7), (8, 0.3), (32, 0.5), (64, 0.7), (64, 0.95), (127, 0.9),
-                                 (128, 0.7), (129, 0.7)])
+                                 (128, 0.7), (129, 0.7), (256, 0.7), (257, 0.5)])
 def test_grouped_llama3_batched(pp, T, p):
     layer_parity(pp, "llama3_8b_batched", T, p)
 
