@@ -20,12 +20,12 @@ from . import build as _build
 F32, BF16, F64 = 0, 1, 2
 RELU, GELU_TANH, SWIGLU = 0, 1, 2
 GATE_SIGMOID, GATE_NONE = 0, 1
-RULE_MIN_PREFIX, RULE_PAPER = 0, 1
+RULE_MIN_PREFIX, RULE_PAPER, RULE_TOPK, RULE_LTE = 0, 1, 2, 3
 OK, ERR_ARG, ERR_NONFINITE = 0, 1, 9
 
 _ACTS = {"relu": RELU, "gelu_tanh": GELU_TANH, "gelu": GELU_TANH, "swiglu": SWIGLU}
 _GATES = {"sigmoid": GATE_SIGMOID, "none": GATE_NONE}
-_RULES = {"min_prefix": RULE_MIN_PREFIX, "paper": RULE_PAPER}
+_RULES = {"min_prefix": RULE_MIN_PREFIX, "paper": RULE_PAPER, "topk": RULE_TOPK, "lte": RULE_LTE}
 
 _lib = None
 _lib_path = None
@@ -112,7 +112,8 @@ def logits(x, Wr):
 
 
 def select(g, p, rule="min_prefix", allow_nonfinite=False):
-    """Softmax, descending order and cumulative-mass cut for each row of g.
+    """Softmax, descending order and cumulative-mass cut for each row of g
+    (rule 'topk': p is k; rule 'lte': p is the sigmoid threshold delta).
 
     Returns (counts[T] int32, ids[T,E] int32 (rank order, -1 padded),
     cum[T,E] fp64 inclusive prefix masses S_i, probs[T,E] fp64).

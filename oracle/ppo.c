@@ -14,6 +14,9 @@
  *   Eq. (tau_thresh_activate)   A = {pi_1} U {pi_i : S_i < tau}     ppo_select
  *   Eq. (ffn), Eq. (moefication_decomp)  FFN_e(x) on expert block e  ppo_sparse_ffn
  *   Eq. (moe_output)            y = sum_{e in A} sigmoid(g_e) FFN_e(x)
+ * and two further activation rules on the same router logits:
+ *   Sec. 4.3 (top-k reconstruction analysis): the first k experts of pi
+ *   Eq. (lte_hard_set)          A = {e : sigmoid(g_e) > delta}  (LTE's rule)
  * Every floating-point operation is done in double precision with plain
  * sequential loops; the inputs (fp32 or bf16) are widened exactly.
  *
@@ -26,6 +29,11 @@
  *    i.e. it also keeps the rank that crosses p.
  *  - p >= 1 selects all E experts under both rules (the warm-up setting
  *    tau_warm = 1.05 of Sec. 3.2 activates every expert); p NaN is an error.
+ *  - TOPK takes k from the same argument p: k = floor(p), at least 1 and
+ *    at most E.  LTE takes delta from p; delta <= 0 selects every expert
+ *    (a sigmoid is positive everywhere, although in fp64 it underflows to 0
+ *    below g = -745), and the set may be empty.  Both list the selected
+ *    experts in the order pi.
  *  - Non-gated FFN variants (Sec. 2.1 says the analysis covers any FFN that
  *    is separable along d_ff): h = relu(x W_up) or h = gelu_tanh(x W_up),
  *    the tanh form of GELU being the GPT-2 one.  No biases (Sec. 2.1).
@@ -51,6 +59,8 @@
 
 #define PPO_RULE_MIN_PREFIX 0
 #define PPO_RULE_PAPER 1
+#define PPO_RULE_TOPK 2
+#define PPO_RULE_LTE 3
 
 #define PPO_OK 0
 #define PPO_ERR_ARG 1
@@ -138,7 +148,7 @@ static int by_rank(const void *pa, const void *pb)
  * For each token: softmax over its E logits (Eq. softmax_prob), the
  * descending order pi (Sec. 3.1), the inclusive prefix masses
  * S_i = sum_{r<=i} p_{pi_r}, and the activated set (Eq. tau_thresh_activate,
- * under the chosen rule).
+ * under the chosen rule; or the top-k / LTE sets, p then carrying k / delta).
  *
  * Outputs: counts[t] = |A|; ids[t][r] = pi_{r+1} for r < |A|, -1 beyond;
  * cum[t][r] = S_{r+1} for all r < E (nullable); probs[t][j] = p_j (nullable).
@@ -148,7 +158,7 @@ static int by_rank(const void *pa, const void *pb)
 int ppo_select(const double *g, int T, int E, double p, int rule, int *counts, int *ids,
                double *cum, double *probs)
 {
-    if (isnan(p) || T < 0 || E <= 0 || (rule != PPO_RULE_MIN_PREFIX && rule != PPO_RULE_PAPER))
+    if (isnan(p) || T < 0 || E <= 0 || rule < PPO_RULE_MIN_PREFIX || rule > PPO_RULE_LTE)
         return PPO_ERR_ARG;
     int status = PPO_OK;
     ranked *order = (ranked *)malloc(sizeof(ranked) * (size_t)E);
@@ -208,6 +218,25 @@ int ppo_select(const double *g, int T, int E, double p, int rule, int *counts, i
                 cum[(size_t)t * E + r] = S;
             if (S < p)
                 below++;
+        }
+
+        if (rule == PPO_RULE_TOPK) {
+            /* the k highest-ranked experts; p carries k */
+            int k = p >= (double)E ? E : (p >= 1.0 ? (int)floor(p) : 1);
+            counts[t] = k;
+            for (int r = 0; r < k; r++)
+                idt[r] = order[r].j;
+            continue;
+        }
+        if (rule == PPO_RULE_LTE) {
+            /* Eq. (lte_hard_set): every expert whose sigmoid score exceeds
+               delta = p, each tested on its own, listed in the order pi */
+            int k = 0;
+            for (int r = 0; r < E; r++)
+                if (p <= 0.0 || ppo_sigmoid(order[r].g) > p)
+                    idt[k++] = order[r].j;
+            counts[t] = k;
+            continue;
         }
 
         int k;

@@ -1,10 +1,12 @@
 """Pins for the CPU oracle: each check ties it to something other than itself.
 
-* hand-worked cases of the paper's definitions (tests/golden/hand_cases.json);
+* hand-worked cases of the paper's definitions (tests/golden/hand_cases.json),
+  including the top-k rule of Sec. 4.3 and LTE's threshold (Eq. lte_hard_set);
 * brute force over all 2^E expert subsets for the cumulative-mass cut
   (Eq. tau_thresh_activate), and an O(E^2) rank-by-comparison restatement;
 * library routines: numpy matmul for Eq. (routing_logits) and the dense FFN,
-  scipy's softmax / expit and torch's GELU / SiLU for the closed forms;
+  scipy's softmax / expit and torch's GELU / SiLU for the closed forms,
+  numpy's lexsort for the top-k order, expit for LTE's set;
 * invariants: the MoEfication identity (Eq. moefication_decomp: all experts
   with unit gates = dense FFN), neuron-permutation invariance (Eq.
   permuted_weights), softmax shift invariance, p >= 1 -> all experts,
@@ -105,6 +107,16 @@ def pin_hand_selection(o):
                 assert got == c[rule], (group["logits"], c["p"], rule, got)
 
 
+def pin_hand_topk_lte(o):
+    """Hand-worked top-k (Sec. 4.3) and LTE (Eq. lte_hard_set) selections."""
+    for group in json.load(open(GOLDEN))["selection_topk_lte"]:
+        g = np.array([group["logits"]], np.float64)
+        for c in group["cases"]:
+            counts, ids, _, _ = o.select(g, c["param"], c["rule"])
+            assert ids[0, :counts[0]].tolist() == c["ids"], (c, ids[0, :counts[0]])
+            assert np.all(ids[0, counts[0]:] == -1)
+
+
 def pin_hand_ffn(o):
     f = json.load(open(GOLDEN))["ffn"]
     x = np.array(f["x"], np.float64)
@@ -192,6 +204,56 @@ def pin_rule_relation(o):
         assert np.all(kp == np.maximum(1, km - 1))
         for t in range(g.shape[0]):
             assert idp[t, :kp[t]].tolist() == idm[t, :kp[t]].tolist()
+
+
+def rank_order(gt):
+    """Descending logit, ties by lower index, by numpy's lexsort."""
+    return np.lexsort((np.arange(gt.shape[0]), -gt))
+
+
+def pin_topk_vs_lexsort(o):
+    """Top-k against a library sort; every kept logit beats every dropped one."""
+    rng = np.random.default_rng(19)
+    E = 48
+    g = np.round(rng.standard_normal((12, E)) * 3.0, 1)  # rounding makes exact ties
+    for k in (0.0, 0.5, 1.0, 2.0, 3.7, 7.0, E - 1.0, float(E), E + 5.0, 1e9):
+        counts, ids, _, _ = o.select(g, k, "topk")
+        want_k = min(E, max(1, int(math.floor(k))))
+        assert np.all(counts == want_k), (k, counts)
+        for t in range(g.shape[0]):
+            ref = rank_order(g[t])
+            assert ids[t, :want_k].tolist() == ref[:want_k].tolist()
+            kept, dropped = g[t, ids[t, :want_k]], np.delete(g[t], ids[t, :want_k])
+            assert dropped.size == 0 or kept.min() >= dropped.max()
+
+
+def pin_lte_vs_expit(o):
+    """LTE's set (Eq. lte_hard_set) against scipy's expit, each expert on its own."""
+    rng = np.random.default_rng(20)
+    E = 40
+    g = rng.standard_normal((16, E)) * 3.0
+    g[0, :4] = 0.0  # sigmoid(0) = 0.5 exactly: excluded at delta = 0.5 (strict >)
+    g[1, :] = -1000.0  # sigmoid underflows to 0 in fp64
+    for delta in (-1.0, 0.0, 1e-30, 0.1, 0.5, 0.73, 0.9, 0.999, 1.0, 2.0):
+        counts, ids, _, _ = o.select(g, delta, "lte")
+        s = scipy.special.expit(g)
+        for t in range(g.shape[0]):
+            if delta <= 0.0:
+                want = set(range(E))  # a sigmoid is positive everywhere
+            else:
+                if np.any(np.abs(s[t] - delta) < 1e-12) and delta != 0.5:
+                    continue
+                want = set(np.nonzero(s[t] > delta)[0].tolist())
+            got = ids[t, :counts[t]].tolist()
+            assert set(got) == want and len(got) == len(want), (delta, t)
+            # listed in the order pi
+            ref = [j for j in rank_order(g[t]).tolist() if j in want]
+            assert got == ref
+            assert np.all(ids[t, counts[t]:] == -1)
+    with pytest.raises(oracle.OracleError):
+        o.select(g, float("nan"), "lte")
+    with pytest.raises(oracle.OracleError):
+        o.select(g, float("nan"), "topk")
 
 
 def pin_special_p(o):
@@ -297,10 +359,10 @@ def pin_permutation_invariance(o):
     np.testing.assert_allclose(y, ref, rtol=1e-11, atol=1e-13)
 
 
-PINS = [pin_hand_selection, pin_hand_ffn, pin_logits_vs_matmul, pin_cum_vs_scipy_softmax,
+PINS = [pin_hand_selection, pin_hand_topk_lte, pin_hand_ffn, pin_logits_vs_matmul, pin_cum_vs_scipy_softmax,
         pin_bruteforce_min_prefix, pin_rank_restatement, pin_rule_relation, pin_special_p,
         pin_shift_invariance_and_huge_logits, pin_nonfinite, pin_activations, pin_dense_identity,
-        pin_masked_dense, pin_permutation_invariance]
+        pin_masked_dense, pin_permutation_invariance, pin_topk_vs_lexsort, pin_lte_vs_expit]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -333,6 +395,11 @@ MUTANTS = {
     "down_neighbour_column": ("yt[j] += w * h * ld(Wd, w_dt, (size_t)j * dff + n);",
                               "yt[j] += w * h * ld(Wd, w_dt, (size_t)j * dff + (n ^ 1));"),
     "gelu_constant": ("0.044715", "0.0447"),
+    "topk_rounds_up": ("(p >= 1.0 ? (int)floor(p) : 1)", "(p >= 1.0 ? (int)ceil(p) : 1)"),
+    "topk_allows_zero": ("(p >= 1.0 ? (int)floor(p) : 1)", "(p >= 1.0 ? (int)floor(p) : 0)"),
+    "lte_not_strict": ("ppo_sigmoid(order[r].g) > p)", "ppo_sigmoid(order[r].g) >= p)"),
+    "lte_delta_le0_not_special": ("if (p <= 0.0 || ppo_sigmoid(order[r].g) > p)", "if (ppo_sigmoid(order[r].g) > p)"),
+    "lte_expert_order": ("idt[k++] = order[r].j;", "idt[k++] = order[E - 1 - r].j;"),
     "expert_block_offset": ("for (int n = e * de; n < (e + 1) * de; n++) {",
                             "for (int n = e * de + (de > 1); n < (e + 1) * de; n++) {"),
 }
