@@ -42,9 +42,14 @@
  *  - Supported shapes: d_expert == 64, d_ff == E * 64, 1 <= E <= 256,
  *    d a multiple of 8 (bf16) or 4 (fp32), 64 <= d <= 8192, T >= 0.
  *    Other shapes return PP_ERR_SHAPE.
- *  - p semantics: p >= 1 activates all E experts (the warm-up setting
- *    tau_warm = 1.05 of Sec. 3.2); p <= 0 activates the top-1 expert only;
- *    NaN returns PP_ERR_INVALID_ARG.
+ *  - p is the parameter of the cut rule (pp_desc.rule); NaN returns
+ *    PP_ERR_INVALID_ARG under every rule.
+ *      MIN_PREFIX, PAPER: the mass budget tau.  p >= 1 activates all E
+ *        experts (the warm-up setting tau_warm = 1.05 of Sec. 3.2); p <= 0
+ *        activates the top-1 expert only.
+ *      TOPK: the expert count k = floor(p), at least 1 and at most E.
+ *      LTE: the score threshold delta; p <= 0 activates all E experts and
+ *        p >= 1 none (counts[t] = 0, y[t] = 0).
  */
 #ifndef PRUNEPATH_H
 #define PRUNEPATH_H
@@ -82,11 +87,20 @@ typedef enum pp_act { PP_ACT_RELU = 0, PP_ACT_GELU_TANH = 1, PP_ACT_SWIGLU = 2 }
    selected expert by 1, the plain decomposition of Eq. (moefication_decomp). */
 typedef enum pp_gate { PP_GATE_SIGMOID = 0, PP_GATE_NONE = 1 } pp_gate;
 
-/* Cut rule on the descending order pi with inclusive prefix masses S_i.
-   MIN_PREFIX: the shortest prefix whose mass reaches p (keeps the rank that
-   crosses p).  PAPER: Eq. (tau_thresh_activate) literally, rank 1 plus every
-   rank with S_i < p.  Whenever S_E >= p, |PAPER| = max(1, |MIN_PREFIX| - 1). */
-typedef enum pp_rule { PP_SEL_MIN_PREFIX = 0, PP_SEL_PAPER = 1 } pp_rule;
+/* Activation rule on the router logits g.  Every rule lists the activated
+   experts in the descending order pi (ties by lower expert index).
+   MIN_PREFIX: the shortest prefix of pi whose mass reaches p (keeps the rank
+   that crosses p).  PAPER: Eq. (tau_thresh_activate) literally, rank 1 plus
+   every rank with S_i < p.  Whenever S_E >= p, |PAPER| =
+   max(1, |MIN_PREFIX| - 1).
+   TOPK: the first k = floor(p) experts of pi, the fixed expert budget of the
+   top-k reconstruction analysis (Sec. 4.3).
+   LTE: every expert with sigmoid(g_e) > p, each expert thresholded on its
+   own (Eq. lte_hard_set, the rule PrunePath is compared with in Sec. 2.3);
+   LTE's own aggregation (Eq. lte_hard_output) is PP_GATE_NONE.  The device
+   takes the same decision on the fp32 logit: g_e >= the smallest fp32 value
+   above ln(p / (1 - p)), a bound the host computes in double precision. */
+typedef enum pp_rule { PP_SEL_MIN_PREFIX = 0, PP_SEL_PAPER = 1, PP_SEL_TOPK = 2, PP_SEL_LTE = 3 } pp_rule;
 
 typedef struct pp_desc {
     int d_model;   /* d                                   */

@@ -17,12 +17,12 @@ PP_ERR_UNSUPPORTED = 10
 PP_F32, PP_BF16 = 0, 1
 PP_ACT_RELU, PP_ACT_GELU_TANH, PP_ACT_SWIGLU = 0, 1, 2
 PP_GATE_SIGMOID, PP_GATE_NONE = 0, 1
-PP_SEL_MIN_PREFIX, PP_SEL_PAPER = 0, 1
+PP_SEL_MIN_PREFIX, PP_SEL_PAPER, PP_SEL_TOPK, PP_SEL_LTE = 0, 1, 2, 3
 
 ACTS = {"relu": PP_ACT_RELU, "gelu_tanh": PP_ACT_GELU_TANH, "gelu": PP_ACT_GELU_TANH,
         "swiglu": PP_ACT_SWIGLU}
 GATES = {"sigmoid": PP_GATE_SIGMOID, "none": PP_GATE_NONE}
-RULES = {"min_prefix": PP_SEL_MIN_PREFIX, "paper": PP_SEL_PAPER}
+RULES = {"min_prefix": PP_SEL_MIN_PREFIX, "paper": PP_SEL_PAPER, "topk": PP_SEL_TOPK, "lte": PP_SEL_LTE}
 DTYPES = {"f32": PP_F32, "bf16": PP_BF16}
 
 

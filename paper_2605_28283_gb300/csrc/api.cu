@@ -106,7 +106,7 @@ pp_status check_desc(const pp_desc* d) {
     if (d->dtype != PP_F32 && d->dtype != PP_BF16) return PP_ERR_DTYPE;
     if (d->act < PP_ACT_RELU || d->act > PP_ACT_SWIGLU) return PP_ERR_INVALID_ARG;
     if (d->gate != PP_GATE_SIGMOID && d->gate != PP_GATE_NONE) return PP_ERR_INVALID_ARG;
-    if (d->rule != PP_SEL_MIN_PREFIX && d->rule != PP_SEL_PAPER) return PP_ERR_INVALID_ARG;
+    if (!rule_known(d->rule)) return PP_ERR_INVALID_ARG;
     if (d->d_expert != kDExpert) return PP_ERR_SHAPE;
     if (d->n_experts < 1 || d->n_experts > kMaxExperts) return PP_ERR_SHAPE;
     if ((long long)d->d_ff != (long long)d->n_experts * kDExpert) return PP_ERR_SHAPE;
@@ -311,6 +311,26 @@ pp_status decode_call(const pp_desc& d, const void* x, int t0, int n, const void
 
 }  // namespace
 
+float rule_kernel_param(int rule, float p, int E) {
+    if (rule == PP_SEL_TOPK) {
+        // k = floor(p) clamped to [1, E]; exact in fp32 since E <= 256
+        if (!(p >= 1.0f)) return 1.0f;
+        return p >= (float)E ? (float)E : std::floor(p);
+    }
+    if (rule == PP_SEL_LTE) {
+        // Eq. (lte_hard_set): sigmoid(g) > delta  <=>  g > t = ln(delta / (1 - delta));
+        // the bound is the smallest float whose value exceeds t
+        if (!(p > 0.0f)) return -INFINITY;
+        if (p >= 1.0f) return INFINITY;
+        const double t = std::log((double)p) - std::log1p(-(double)p);
+        float f = (float)t;
+        while ((double)f <= t) f = std::nextafter(f, INFINITY);
+        while ((double)std::nextafter(f, -INFINITY) > t) f = std::nextafter(f, -INFINITY);
+        return f;
+    }
+    return p;
+}
+
 TensorMapEncodeFn tensor_map_encoder() {
     static TensorMapEncodeFn fn = nullptr;
     static std::once_flag once;
@@ -353,7 +373,8 @@ pp_status pp_select(const pp_desc* desc, const float* logits, int T, float p, co
     PP_TRY(check_device());
     if (T == 0) return PP_OK;
     const Ws w = ws_views(*desc, T, ws);
-    return cuda_status(select_launch(logits, T, desc->n_experts, p, desc->rule, desc->gate, out->ids,
+    const float kp = rule_kernel_param(desc->rule, p, desc->n_experts);
+    return cuda_status(select_launch(logits, T, desc->n_experts, kp, desc->rule, desc->gate, out->ids,
                                      out->counts, out->gates, &w.ctrl->status,
                                      static_cast<cudaStream_t>(stream)));
 }
@@ -371,17 +392,18 @@ pp_status pp_route(const pp_desc* desc, const void* x, int T, const void* W_r, f
     if (T == 0) return PP_OK;
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     const Ws w = ws_views(*desc, T, ws);
+    const float kp = rule_kernel_param(desc->rule, p, desc->n_experts);
     if (use_grouped(*desc, T)) {
-        const GroupedArgs a = grouped_args(*desc, T, ws, x, W_r, nullptr, nullptr, nullptr, p, *out, nullptr);
+        const GroupedArgs a = grouped_args(*desc, T, ws, x, W_r, nullptr, nullptr, nullptr, kp, *out, nullptr);
         return cuda_status(grouped_route(a, st));
     }
     const int ts = decode_ts_limit(*desc);
     if (ts == 0) return PP_ERR_SHAPE;
     if (T <= ts)
-        return decode_call(*desc, x, 0, T, W_r, nullptr, nullptr, nullptr, p, out, true, false, nullptr, w, st);
+        return decode_call(*desc, x, 0, T, W_r, nullptr, nullptr, nullptr, kp, out, true, false, nullptr, w, st);
     float* lg = out->logits ? out->logits : w.logits;
     PP_TRY(cuda_status(router_launch(desc->dtype, x, T, desc->d_model, W_r, desc->n_experts, lg, st)));
-    return cuda_status(select_launch(lg, T, desc->n_experts, p, desc->rule, desc->gate, out->ids, out->counts,
+    return cuda_status(select_launch(lg, T, desc->n_experts, kp, desc->rule, desc->gate, out->ids, out->counts,
                                      out->gates, &w.ctrl->status, st));
 }
 
@@ -428,18 +450,19 @@ pp_status pp_layer(const pp_desc* desc, const void* x, int T, const void* W_r, c
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     const Ws w = ws_views(*desc, T, ws);
     pp_selection s = sel_out ? *sel_out : pp_selection{w.ids, w.counts, w.gates, nullptr};
+    const float kp = rule_kernel_param(desc->rule, p, desc->n_experts);
     if (use_grouped(*desc, T)) {
-        const GroupedArgs a = grouped_args(*desc, T, ws, x, W_r, W_gate, W_up, W_down, p, s, y);
+        const GroupedArgs a = grouped_args(*desc, T, ws, x, W_r, W_gate, W_up, W_down, kp, s, y);
         PP_TRY(cuda_status(grouped_route(a, st)));
         return cuda_status(grouped_ffn(a, device_info().sms, st));
     }
     const int ts = decode_ts_limit(*desc);
     if (ts == 0) return PP_ERR_SHAPE;
     if (T <= ts)
-        return decode_call(*desc, x, 0, T, W_r, W_gate, W_up, W_down, p, sel_out, true, true, y, w, st);
+        return decode_call(*desc, x, 0, T, W_r, W_gate, W_up, W_down, kp, sel_out, true, true, y, w, st);
     float* lg = s.logits ? s.logits : w.logits;
     PP_TRY(cuda_status(router_launch(desc->dtype, x, T, desc->d_model, W_r, desc->n_experts, lg, st)));
-    PP_TRY(cuda_status(select_launch(lg, T, desc->n_experts, p, desc->rule, desc->gate, s.ids, s.counts, s.gates,
+    PP_TRY(cuda_status(select_launch(lg, T, desc->n_experts, kp, desc->rule, desc->gate, s.ids, s.counts, s.gates,
                                      &w.ctrl->status, st)));
     for (int t0 = 0; t0 < T; t0 += ts) {
         const int n = std::min(ts, T - t0);

@@ -79,7 +79,7 @@ pp_status check_args(const pp_desc* d, int T, const void* x, const void* Wr, con
     if (d->dtype != PP_F32 && d->dtype != PP_BF16) return PP_ERR_DTYPE;
     if (d->act < PP_ACT_RELU || d->act > PP_ACT_SWIGLU) return PP_ERR_INVALID_ARG;
     if (d->gate != PP_GATE_SIGMOID && d->gate != PP_GATE_NONE) return PP_ERR_INVALID_ARG;
-    if (d->rule != PP_SEL_MIN_PREFIX && d->rule != PP_SEL_PAPER) return PP_ERR_INVALID_ARG;
+    if (!pp::rule_known(d->rule)) return PP_ERR_INVALID_ARG;
     if (d->d_expert != pp::kDExpert || d->n_experts < 1 || d->n_experts > pp::kMaxExperts) return PP_ERR_SHAPE;
     if ((long long)d->d_ff != (long long)d->n_experts * pp::kDExpert) return PP_ERR_SHAPE;
     const int vec = d->dtype == PP_BF16 ? 8 : 4;
@@ -163,7 +163,7 @@ extern "C" pp_status pp_layer_noalloc(const pp_desc* desc, const void* x, int T,
     a.act = d.act;
     a.gate = d.gate;
     a.rule = d.rule;
-    a.p = p;
+    a.p = pp::rule_kernel_param(d.rule, p, d.n_experts);
     a.do_route = 1;
     a.do_ffn = 1;
     a.R6 = plan.R6;

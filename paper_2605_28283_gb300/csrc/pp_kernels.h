@@ -14,6 +14,16 @@
 
 namespace pp {
 
+// ---------------------------------------------------------------- rules
+// Whether `rule` is one of the pp_rule values.
+inline bool rule_known(int rule) { return rule >= PP_SEL_MIN_PREFIX && rule <= PP_SEL_LTE; }
+
+// The rule parameter p (not NaN) in the form the selection kernels take:
+// the mass budget for MIN_PREFIX / PAPER, the count k in [1, E] for TOPK,
+// and for LTE the smallest fp32 logit g with sigmoid(g) > p (-inf for
+// p <= 0: every logit; +inf for p >= 1: none).
+float rule_kernel_param(int rule, float p, int E);
+
 // ---------------------------------------------------------------- decode
 struct DecodeArgs {
     CUtensorMap tmap_down;  // W_down [d][d_ff], box {64, R6}; must stay first (64-byte aligned)

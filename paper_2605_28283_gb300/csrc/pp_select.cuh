@@ -7,7 +7,8 @@
 // strides < S, shuffles otherwise), then forms the max-shifted fp32
 // exponentials in rank order and their inclusive prefix sums in fp64.  The
 // cut compares each prefix with p * Z in fp64.  After the sort lane l holds
-// ranks l*S .. l*S+S-1 in key[0..S-1].
+// ranks l*S .. l*S+S-1 in key[0..S-1].  The same order serves the top-k rule
+// (Sec. 4.3) and LTE's threshold rule (Eq. lte_hard_set).
 #pragma once
 
 #include "pp_common.cuh"
@@ -82,6 +83,11 @@ PP_DEVINL void warp_bitonic_sort(unsigned long long (&key)[S]) {
     }
 }
 
+// The rule parameter as the kernels take it (rule_kernel_param on the host):
+// MIN_PREFIX / PAPER the mass budget p; TOPK the count k (an integer in
+// [1, E]); LTE the smallest activated fp32 logit (Eq. lte_hard_set:
+// sigmoid(g) > delta  <=>  g > ln(delta / (1 - delta))).
+
 // Selection of one token by one warp.  `load(j)` returns logit j (j < E).
 // Returns the activated count k (warp-uniform); 0 when a logit is not finite
 // (then *finite_out = false).  key[] is left sorted (see file comment).
@@ -106,6 +112,14 @@ PP_DEVINL int warp_select(Load load, int E, float p, int rule, unsigned long lon
     if (!all_finite) return 0;
 
     warp_bitonic_sort<S>(key);
+
+    if (rule == PP_SEL_TOPK) return min(E, (int)p);  // the first k ranks
+    if (rule == PP_SEL_LTE) {  // the logits at or above the bound form a prefix of the order
+        int n = 0;
+#pragma unroll
+        for (int s = 0; s < S; s++) n += __popc(__ballot_sync(kFull, lane * S + s < E && key_logit(key[s]) >= p));
+        return n;
+    }
 
     const float m = key_logit(__shfl_sync(kFull, key[0], 0));  // rank 1 holds max g
     double pre[S];
@@ -161,15 +175,25 @@ PP_DEVINL float gate_of(int gate_mode, unsigned long long k) {
 //   PAPER:      j activated <=> A_j == 0 (rank 0)  or  A_j + U_j <  p Z
 // (the top expert has e = 1, U = 2^31 > 0, so A_j == 0 exactly at rank 0;
 // A is non-decreasing along the order, so both sets are prefixes of it).
+// TOPK counts with U = 1 for every expert, so A_j is the rank of j:
+//   TOPK:       j activated <=> A_j < k
+// and LTE needs no count at all:
+//   LTE:        j activated <=> g_j >= the bound.
 
 struct CtaSelScratch {
-    // order keys D[0..255] and fixed-point exponentials U[256..511] (e * 2^31);
-    // after the count, the same bytes hold the activated (D, index) keys
+    // order keys D[0..255] and fixed-point exponentials U[256..511] (e * 2^31)
+    // for the top-k count; the (D, index) keys of the mass-cut candidates;
+    // after the count, the activated (D, index) keys
     __align__(16) uint32_t DU[2 * kMaxExperts];
     float fred[8];
     unsigned long long ured[8];
     int wcnt[8];
+    __align__(16) uint32_t cu[kMaxExperts];  // U of each compacted candidate (keys in DU)
+    uint8_t flag[kMaxExperts];               // activated experts of the candidate path
+    int ncand;
 };
+
+constexpr int kDecSelThreads = 256;  // the CTA selection runs on 8 warps
 
 PP_DEVINL uint32_t desc_key(float g) {
     unsigned u = __float_as_uint(g);
@@ -206,6 +230,7 @@ PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, bool want_rank,
     const float g = valid ? load(j) : -INFINITY;
     *gval = g;
     *rank = -1;
+    sc.flag[j] = 0;  // read back after the count (a later barrier orders it)
     const bool fin = !valid || isfinite(g);
     if (!__syncthreads_and(fin)) {
         if (j == 0) record_status(status, PP_ERR_NONFINITE);
@@ -225,12 +250,20 @@ PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, bool want_rank,
     }
     // fixed-point exponentials and their sum Z
     const float e = valid ? expf(g - m) : 0.0f;
-    const uint32_t U = valid ? __float2uint_rn(e * 2147483648.0f) : 0u;
+    const uint32_t U = valid ? (rule == PP_SEL_TOPK ? 1u : __float2uint_rn(e * 2147483648.0f)) : 0u;
     const uint32_t D = valid ? desc_key(g) : 0xffffffffu;  // a finite logit never gives all ones
     uint32_t* sD = sc.DU;
     uint32_t* sU = sc.DU + kMaxExperts;
-    sD[j] = D;
-    sU[j] = U;
+    unsigned long long* sK = reinterpret_cast<unsigned long long*>(sc.DU);
+    if (rule == PP_SEL_TOPK) {
+        sD[j] = D;
+        sU[j] = U;
+    } else {
+        // padding of the candidate list (a key that is never ahead)
+        sK[j] = ~0ull;
+        sc.cu[j] = 0u;
+        if (j == 0) sc.ncand = 0;
+    }
     unsigned long long z = U;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(kFull, z, o);
@@ -242,59 +275,118 @@ PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, bool want_rank,
         const ulonglong2 a = v[0], b = v[1], c = v[2], d2 = v[3];
         Z = (a.x + a.y) + (b.x + b.y) + (c.x + c.y) + (d2.x + d2.y);
     }
-    // exclusive prefix mass: the exponentials of the experts ahead, four
-    // independent accumulator chains; candidates [0, w0) have a lower index
-    // than every thread of this warp, [w0, w1) are the warp's own experts,
-    // [w1, E) have a higher index
-    unsigned long long m0 = 0, m1 = 0, m2 = 0, m3 = 0;
-    const int w0 = warp * 32, w1 = min(E, w0 + 32);
-    if (w0 < E) {  // warps without an expert skip the count
-        const uint32_t thrB = D + 1u, thrA = D;
-        // candidates [i0, i1) against threshold th (or, in the warp's own
-        // range, th for index >= j and th + 1 below j); 16 candidates are
-        // loaded before any of them is compared, so the shared-memory
-        // latency is paid once per 16
-        auto accum = [&](int i0, int i1, uint32_t th, bool own) {
-            int i = i0;
-            for (; i + 16 <= i1; i += 16) {
-                uint4 d4[4], u4[4];
+    bool on = false, counted = false, filtered = false;
+    if (rule == PP_SEL_LTE) {
+        on = counted = valid && g >= p;
+    } else if (rule != PP_SEL_TOPK && p >= 1.0f) {
+        on = counted = valid;  // every expert (warm-up reading)
+    } else if (rule == PP_SEL_TOPK) {
+        // exclusive rank by counting, four independent accumulator chains;
+        // candidates [0, w0) have a lower index than every thread of this
+        // warp, [w0, w1) are the warp's own experts, [w1, E) have a higher
+        // index
+        unsigned long long m0 = 0, m1 = 0, m2 = 0, m3 = 0;
+        const int w0 = warp * 32, w1 = min(E, w0 + 32);
+        if (w0 < E) {  // warps without an expert skip the count
+            const uint32_t thrB = D + 1u, thrA = D;
+            // candidates [i0, i1) against threshold th (or, in the warp's own
+            // range, th for index >= j and th + 1 below j); 16 candidates are
+            // loaded before any of them is compared, so the shared-memory
+            // latency is paid once per 16
+            auto accum = [&](int i0, int i1, uint32_t th, bool own) {
+                int i = i0;
+                for (; i + 16 <= i1; i += 16) {
+                    uint4 d4[4], u4[4];
 #pragma unroll
-                for (int k = 0; k < 4; k++) {
-                    d4[k] = *reinterpret_cast<const uint4*>(&sD[i + 4 * k]);
-                    u4[k] = *reinterpret_cast<const uint4*>(&sU[i + 4 * k]);
-                }
+                    for (int k = 0; k < 4; k++) {
+                        d4[k] = *reinterpret_cast<const uint4*>(&sD[i + 4 * k]);
+                        u4[k] = *reinterpret_cast<const uint4*>(&sU[i + 4 * k]);
+                    }
 #pragma unroll
-                for (int k = 0; k < 4; k++) {
-                    const int b = i + 4 * k;
-                    const uint32_t t0 = own && b + 0 < j ? th + 1u : th, t1 = own && b + 1 < j ? th + 1u : th;
-                    const uint32_t t2 = own && b + 2 < j ? th + 1u : th, t3 = own && b + 3 < j ? th + 1u : th;
-                    m0 += d4[k].x < t0 ? (unsigned long long)u4[k].x : 0ull;
-                    m1 += d4[k].y < t1 ? (unsigned long long)u4[k].y : 0ull;
-                    m2 += d4[k].z < t2 ? (unsigned long long)u4[k].z : 0ull;
-                    m3 += d4[k].w < t3 ? (unsigned long long)u4[k].w : 0ull;
+                    for (int k = 0; k < 4; k++) {
+                        const int b = i + 4 * k;
+                        const uint32_t t0 = own && b + 0 < j ? th + 1u : th, t1 = own && b + 1 < j ? th + 1u : th;
+                        const uint32_t t2 = own && b + 2 < j ? th + 1u : th, t3 = own && b + 3 < j ? th + 1u : th;
+                        m0 += d4[k].x < t0 ? (unsigned long long)u4[k].x : 0ull;
+                        m1 += d4[k].y < t1 ? (unsigned long long)u4[k].y : 0ull;
+                        m2 += d4[k].z < t2 ? (unsigned long long)u4[k].z : 0ull;
+                        m3 += d4[k].w < t3 ? (unsigned long long)u4[k].w : 0ull;
+                    }
                 }
-            }
-            for (; i < i1; i++) m0 += sD[i] < (own && i < j ? th + 1u : th) ? (unsigned long long)sU[i] : 0ull;
-        };
-        accum(0, w0, thrB, false);
-        accum(w0, w1, thrA, true);
-        accum(w1, E, thrA, false);
-    }
-    const unsigned long long ahead = (m0 + m1) + (m2 + m3);
-    bool on;
-    if (p >= 1.0f) {
-        on = valid;
+                for (; i < i1; i++) m0 += sD[i] < (own && i < j ? th + 1u : th) ? (unsigned long long)sU[i] : 0ull;
+            };
+            accum(0, w0, thrB, false);
+            accum(w0, w1, thrA, true);
+            accum(w1, E, thrA, false);
+        }
+        const unsigned long long ahead = (m0 + m1) + (m2 + m3);
+        on = counted = valid && ahead < (unsigned long long)(int)p;
     } else {
-        const long long thr = prefix_threshold(p, Z);
-        const unsigned long long mass = rule == PP_SEL_PAPER ? ahead + U : ahead;
-        on = valid && (ahead == 0ull || (thr >= 0 && mass <= (unsigned long long)thr));
+        // Cumulative-mass cut.  Only experts near the top of the order can
+        // be activated: the mass at or behind an activated j exceeds
+        // (1 - p) Z and consists of at most E exponentials no larger than
+        // e_j (up to the 2-ulp error of expf), so e_j > (1 - p) Z / E.  The
+        // candidates are the experts with g_j - m >= ln of half that bound
+        // (a slack of ln 2 for the roundings); the test is monotone in g, so
+        // they form a prefix of the order, every expert ahead of a
+        // candidate is one, and a candidate's exclusive prefix mass A_j is
+        // summed over the candidates alone.  Below a bound of 20 * 2^-31
+        // every expert is a candidate.
+        filtered = true;
+        const float Bm = (1.0f - fmaxf(p, 0.0f)) * ((float)Z * (1.0f / 2147483648.0f)) / (float)E;
+        const float Lc = Bm >= 20.0f / 2147483648.0f ? logf(0.5f * Bm) : -INFINITY;
+        const bool cand = valid && (g - m) >= Lc;
+        // compaction in arrival order through a warp-aggregated shared
+        // counter; the key (D, index) carries the tie-break, and the slots
+        // past the last candidate keep the padding written before the
+        // previous barrier
+        const unsigned bal = __ballot_sync(kFull, cand);
+        int wbase = 0;
+        if (lane == 0 && bal) wbase = atomicAdd(&sc.ncand, __popc(bal));
+        wbase = __shfl_sync(kFull, wbase, 0);
+        if (cand) {
+            const int q = wbase + __popc(bal & ((1u << lane) - 1u));
+            sK[q] = ((unsigned long long)D << 32) | (unsigned)j;
+            sc.cu[q] = U;
+        }
+        __syncthreads();
+        const int nc = sc.ncand;
+        // nt threads per candidate (aligned lane groups), each summing a
+        // contiguous run of the candidates, four at a time
+        int nt = 16;
+        while (nt > 1 && nc * nt > kDecSelThreads) nt >>= 1;
+        const int q = j / nt, part = j % nt;
+        unsigned long long a0 = 0ull, a1 = 0ull;
+        if (q < nc) {
+            const unsigned long long Kq = sK[q];
+            const int nv = (nc + 3) >> 2, per = (nv + nt - 1) / nt;
+            const int v1 = min(nv, (part + 1) * per);
+            const ulonglong2* k2 = reinterpret_cast<const ulonglong2*>(sK);
+            const uint4* u4p = reinterpret_cast<const uint4*>(sc.cu);
+            for (int v = part * per; v < v1; v++) {
+                const ulonglong2 ka = k2[2 * v], kb = k2[2 * v + 1];
+                const uint4 u4 = u4p[v];
+                a0 += ka.x < Kq ? (unsigned long long)u4.x : 0ull;
+                a1 += ka.y < Kq ? (unsigned long long)u4.y : 0ull;
+                a0 += kb.x < Kq ? (unsigned long long)u4.z : 0ull;
+                a1 += kb.y < Kq ? (unsigned long long)u4.w : 0ull;
+            }
+        }
+        unsigned long long a = a0 + a1;
+        for (int o = 1; o < nt; o <<= 1) a += __shfl_xor_sync(kFull, a, o);
+        if (q < nc && part == 0) {
+            const long long thr = prefix_threshold(p, Z);
+            const unsigned long long mass = rule == PP_SEL_PAPER ? a + sc.cu[q] : a;
+            counted = a == 0ull || (thr >= 0 && mass <= (unsigned long long)thr);
+            if (counted) sc.flag[(unsigned)sK[q] & 0xffu] = 1;
+        }
     }
+    const int k = __syncthreads_count(counted);  // also: every thread is done reading sD, sU
+    if (filtered) on = valid && sc.flag[j] != 0;
     *sel = on;
-    const int k = __syncthreads_count(on);  // also: every thread is done reading sD, sU
     if (want_rank) {
         // rank of an activated expert = activated keys (D, index) below its
         // own; the activated keys are compacted into the scratch first
-        unsigned long long* sK = reinterpret_cast<unsigned long long*>(sc.DU);
         const unsigned long long key = ((unsigned long long)D << 32) | (unsigned)j;
         const unsigned bal = __ballot_sync(kFull, on);
         if (lane == 0) sc.wcnt[warp] = __popc(bal);

@@ -1,8 +1,8 @@
 """GPU parity: the CUDA library (through its C ABI) against the CPU oracle.
 
 Cases cover all five workload shapes (tiny ReLU fp32, GPT-2-medium GELU,
-Llama-2-7B / Llama-3-8B SwiGLU decode, Llama-2-13B SwiGLU), both cut rules,
-both gate modes, p from <= 0 to >= 1, token counts that exercise the fused
+Llama-2-7B / Llama-3-8B SwiGLU decode, Llama-2-13B SwiGLU), the two
+cumulative-mass cut rules plus top-k and LTE's threshold, both gate modes, p from <= 0 to >= 1, token counts that exercise the fused
 decode kernel (T <= 4 bf16 / 8 fp32), its token slices and the stand-alone
 router + selection kernels, plus the degenerate inputs (ties, signed zeros,
 huge and non-finite logits, T = 0).
@@ -87,6 +87,38 @@ def test_layer_rules_gates(pp, rule, gate, p):
     layer_parity(pp, "llama2_7b_decode", 3, p, rule, gate, d=512, E=40)
 
 
+# Top-k (Sec. 4.3) and LTE's threshold (Eq. lte_hard_set) on the same
+# kernels: the fused decode kernel (T <= 4 bf16, fp32 slices), the router +
+# selection kernels and the grouped tensor-core path (bf16, T >= 5).  LTE at
+# delta = 0.999 leaves some tokens without any expert (y = 0).
+RULE_CASES = [("topk", 1.0), ("topk", 2.5), ("topk", 7.0), ("topk", 500.0), ("lte", -1.0), ("lte", 0.5),
+              ("lte", 0.9), ("lte", 0.999), ("lte", 1.0)]
+
+
+@pytest.mark.parametrize("rule,p", RULE_CASES)
+@pytest.mark.parametrize("gate", ["sigmoid", "none"])
+def test_layer_topk_lte_decode(pp, rule, p, gate):
+    layer_parity(pp, "llama2_7b_decode", 3, p, rule, gate, d=512, E=40)
+
+
+@pytest.mark.parametrize("rule,p", [("topk", 3.0), ("lte", 0.95), ("lte", 0.999)])
+@pytest.mark.parametrize("name,T", [("tiny_relu_f32", 64), ("gpt2m_gelu_bf16", 16), ("llama3_8b_batched", 8),
+                                    ("llama3_8b_batched", 64), ("llama2_13b_prefill", 300)])
+def test_layer_topk_lte_batched(pp, name, T, rule, p):
+    layer_parity(pp, name, T, p, rule, "none" if rule == "lte" else "sigmoid")
+
+
+def test_layer_lte_empty_tokens(pp):
+    """Tokens whose every score stays at or below delta get no expert and y = 0."""
+    for T in (2, 37):
+        w, L = layer_inputs("llama2_7b_decode", T, d=512, E=40)
+        counts, ids, logits, y, status = run_layer(pp, w, L, 1.0, "lte", "none")
+        assert status == pp.PP_OK
+        assert np.all(counts == 0) and np.all(ids == -1) and np.all(y == 0.0)
+        counts, ids, logits, y, status = run_layer(pp, w, L, -2.0, "lte", "none")
+        assert status == pp.PP_OK and np.all(counts == w.n_experts)
+
+
 @pytest.mark.parametrize("d,E,T", [(64, 1, 2), (128, 3, 5), (200, 33, 4), (2048, 256, 3), (8192, 100, 1)])
 def test_layer_odd_shapes(pp, d, E, T):
     layer_parity(pp, "llama3_8b_batched", T, 0.8, d=d, E=E)
@@ -157,6 +189,25 @@ def test_route(pp, name, T, rule):
         assert np.all(gates[t, k:] == 0)
 
 
+@pytest.mark.parametrize("name,T", [("llama2_7b_decode", 1), ("gpt2m_gelu_bf16", 4), ("tiny_relu_f32", 64),
+                                    ("llama3_8b_batched", 64), ("llama2_13b_prefill", 300)])
+@pytest.mark.parametrize("rule,p", [("topk", 4.0), ("lte", 0.9)])
+def test_route_topk_lte(pp, name, T, rule, p):
+    import torch
+    w, L = layer_inputs(name, T)
+    desc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act, "sigmoid", rule)
+    ws = pp.alloc_workspace(desc, T)
+    sel = pp.Selection.empty(T, w.n_experts, "cuda")
+    pp.pp_route(desc, dev(L.x), T, dev(L.Wr), p, sel, ws)
+    torch.cuda.synchronize()
+    assert pp.pp_get_device_status(ws) == pp.PP_OK
+    g_ref = oracle.logits(L.x, L.Wr)
+    lg = to_host(sel.logits)
+    assert np.all(np.abs(lg - g_ref) <= logit_tolerance(L.x, L.Wr))
+    eps = np.abs(lg - g_ref).max(axis=1)
+    check_route_selection(to_host(sel.counts), to_host(sel.ids), g_ref, eps, p, rule)
+
+
 # --------------------------------------------------------------- pp_select
 def select_gpu(pp, logits, p, rule, gate="sigmoid"):
     import torch
@@ -191,6 +242,43 @@ def test_select_bit_exact(pp, E, rule, T):
     assert total_boundary <= max(2, T * 7 * 0.01)
 
 
+@pytest.mark.parametrize("T", [40, 2000])
+@pytest.mark.parametrize("E", [1, 5, 33, 64, 172, 224, 256])
+@pytest.mark.parametrize("rule", ["topk", "lte"])
+def test_select_topk_lte_bit_exact(pp, E, rule, T):
+    """Top-k is exact (no boundary); LTE is exact except scores within 1e-6 of delta."""
+    logits = wl.host_logits(T, E, std=3.0, seed=E + 1)
+    params = (0.0, 0.5, 1.0, 2.0, 5.5, E - 1.0, float(E), 1e9) if rule == "topk" else \
+        (-1.0, 0.0, 0.05, 0.3, 0.5, 0.8, 0.97, 0.9999, 1.0, 3.0)
+    nb = 0
+    for p in params:
+        pf = f32(p)
+        counts, ids, gates, status = select_gpu(pp, logits, pf, rule)
+        assert status == pp.PP_OK
+        g = logits.astype(np.float64)
+        nb += check_select_exact(counts, ids, g, pf, rule)
+        for t in range(0, T, 97):
+            k = counts[t]
+            ref = 1.0 / (1.0 + np.exp(-g[t, ids[t, :k]]))
+            np.testing.assert_allclose(gates[t, :k], ref, rtol=2e-6, atol=1e-30)
+            assert np.all(gates[t, k:] == 0)
+    assert nb <= max(2, T * len(params) * 0.01)
+
+
+def test_select_lte_exact_threshold(pp):
+    """A logit exactly at ln(delta / (1 - delta)) is not activated (strict >),
+    the next float above it is: sigmoid(0) = 0.5 exactly."""
+    E = 8
+    logits = np.zeros((3, E), np.float32)
+    logits[1, 3] = np.nextafter(np.float32(0.0), np.float32(1.0))
+    logits[2, :] = np.float32(-0.0)
+    logits[2, 5] = np.float32(1e-3)
+    counts, ids, gates, status = select_gpu(pp, logits, 0.5, "lte")
+    assert status == pp.PP_OK
+    assert counts.tolist() == [0, 1, 1]
+    assert ids[1, 0] == 3 and ids[2, 0] == 5
+
+
 @pytest.mark.parametrize("T", [16, 500])
 def test_select_ties_and_zeros(pp, T):
     rng = np.random.default_rng(5)
@@ -201,9 +289,10 @@ def test_select_ties_and_zeros(pp, T):
     logits[2, :] = np.float32(-1e4)
     logits[2, 7] = np.float32(1e4)
     logits[3, :] = np.linspace(30, -30, E).astype(np.float32)
-    for rule in ("min_prefix", "paper"):
+    for rule, ps in (("min_prefix", (0.1, 0.5, 0.75, 0.999, 1.0)), ("paper", (0.1, 0.5, 0.75, 0.999, 1.0)),
+                     ("topk", (1.0, 3.0, 50.0)), ("lte", (0.5, 0.9))):
         for gate in ("sigmoid", "none"):
-            for p in (0.1, 0.5, 0.75, 0.999, 1.0):
+            for p in ps:
                 pf = f32(p)
                 counts, ids, gates, status = select_gpu(pp, logits, pf, rule, gate)
                 assert status == pp.PP_OK
