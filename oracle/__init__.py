@@ -57,6 +57,8 @@ def load(path: str = None):
     lib.ppo_sparse_ffn.argtypes = [_P, _I, _I, _I, _I, _I, _I, _I, _P, _P, _P, _I, _P, _P, _P, _P]
     lib.ppo_dense_ffn.restype = _I
     lib.ppo_dense_ffn.argtypes = [_P, _I, _I, _I, _I, _I, _P, _P, _P, _I, _P]
+    lib.ppo_router_stats.restype = _I
+    lib.ppo_router_stats.argtypes = [_P, _I, _I, _D, _P]
     lib.ppo_layer.restype = _I
     lib.ppo_layer.argtypes = [_P, _I, _I, _I, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _I, _P,
                               _P, _P, _P]
@@ -169,6 +171,20 @@ def dense_ffn(x, Wg, Wu, Wd, act_kind="swiglu"):
     if s:
         raise OracleError(s, "ppo_dense_ffn")
     return y
+
+
+def router_stats(g, eps=1e-9):
+    """Eq. (entropy_loss), Eq. (load_balance_loss) and the gate-magnitude
+    term L_gate over the batch of logits g [B, E].  Returns (L_ent, L_bal,
+    L_gate) as floats."""
+    lib = load()
+    g = np.ascontiguousarray(g, dtype=np.float64)
+    T, E = g.shape
+    out = np.empty(3, np.float64)
+    s = lib.ppo_router_stats(_ptr(g), T, E, float(eps), _ptr(out))
+    if s:
+        raise OracleError(s, "ppo_router_stats")
+    return float(out[0]), float(out[1]), float(out[2])
 
 
 def layer(x, Wr, Wg, Wu, Wd, p, act_kind="swiglu", gate="sigmoid", rule="min_prefix"):

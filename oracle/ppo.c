@@ -17,6 +17,8 @@
  * and two further activation rules on the same router logits:
  *   Sec. 4.3 (top-k reconstruction analysis): the first k experts of pi
  *   Eq. (lte_hard_set)          A = {e : sigmoid(g_e) > delta}  (LTE's rule)
+ * and the router statistics of the training objective (forward values):
+ *   Eq. (entropy_loss), Eq. (load_balance_loss), L_gate (Sec. 4.2.3)          ppo_router_stats
  * Every floating-point operation is done in double precision with plain
  * sequential loops; the inputs (fp32 or bf16) are widened exactly.
  *
@@ -351,4 +353,71 @@ int ppo_layer(const void *x, int x_dt, int T, int d, int E, int de, int act, int
     int s2 = ppo_sparse_ffn(x, x_dt, T, d, E, de, act, gate_mode, Wg, Wu, Wd, w_dt, counts, ids,
                             g, y);
     return s != PPO_OK ? s : s2;
+}
+
+/* ---- router statistics (Sec. 3.2 and Sec. 4.2.3) --------------------------- */
+
+/*
+ * Over a batch of B = T tokens with router logits g[t][j] and softmax
+ * probabilities p_tj (Eq. softmax_prob):
+ *   out[0] = L_ent  = -(1/B) sum_t sum_j p_tj log(p_tj + eps)   (Eq. entropy_loss)
+ *   out[1] = L_bal  = E sum_j ((1/B) sum_t p_tj)^2              (Eq. load_balance_loss)
+ *   out[2] = L_gate = (1/(B E)) sum_t sum_j sigmoid(g_tj)        (the gate-magnitude
+ *            regulariser of the instruction-tuning experiments)
+ * Forward values only.  Returns PPO_ERR_ARG for T < 1 or E < 1 and
+ * PPO_ERR_NONFINITE if a logit is not finite (out is then NaN).
+ */
+int ppo_router_stats(const double *g, int T, int E, double eps, double *out)
+{
+    if (T < 1 || E < 1 || isnan(eps))
+        return PPO_ERR_ARG;
+    double *colsum = (double *)calloc((size_t)E, sizeof(double));
+    double *prob = (double *)malloc(sizeof(double) * (size_t)E);
+    if (!colsum || !prob) {
+        free(colsum);
+        free(prob);
+        return PPO_ERR_ARG;
+    }
+    double ent = 0.0, gate = 0.0;
+    int status = PPO_OK;
+    for (int t = 0; t < T; t++) {
+        const double *gt = g + (size_t)t * E;
+        int finite = 1;
+        for (int j = 0; j < E; j++)
+            finite &= isfinite(gt[j]) ? 1 : 0;
+        if (!finite) {
+            status = PPO_ERR_NONFINITE;
+            break;
+        }
+        double m = gt[0];
+        for (int j = 1; j < E; j++)
+            if (gt[j] > m)
+                m = gt[j];
+        double Z = 0.0;
+        for (int j = 0; j < E; j++) {
+            prob[j] = exp(gt[j] - m);
+            Z += prob[j];
+        }
+        for (int j = 0; j < E; j++) {
+            const double pj = prob[j] / Z;
+            ent -= pj * log(pj + eps);
+            colsum[j] += pj;
+            gate += ppo_sigmoid(gt[j]);
+        }
+    }
+    if (status == PPO_OK) {
+        double bal = 0.0;
+        for (int j = 0; j < E; j++) {
+            const double f = colsum[j] / (double)T;
+            bal += f * f;
+        }
+        out[0] = ent / (double)T;
+        out[1] = (double)E * bal;
+        out[2] = gate / ((double)T * (double)E);
+    } else {
+        out[0] = out[1] = out[2] = NAN;
+    }
+    free(colsum);
+    free(prob);
+    return status;
 }

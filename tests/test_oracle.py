@@ -256,6 +256,40 @@ def pin_lte_vs_expit(o):
         o.select(g, float("nan"), "topk")
 
 
+def pin_router_stats(o):
+    """Eq. entropy_loss, Eq. load_balance_loss and L_gate: closed forms and a
+    scipy restatement."""
+    E, B, eps = 16, 5, 1e-9
+    # equal logits: p = 1/E everywhere
+    ent, bal, gate = o.router_stats(np.full((B, E), 0.7), eps)
+    assert abs(ent - (-math.log(1.0 / E + eps))) <= 1e-14 * math.log(E)
+    assert abs(bal - 1.0) <= 1e-14
+    assert abs(gate - scipy.special.expit(0.7)) <= 1e-15
+    # one-hot tokens (exp underflows to exactly 0): all on expert 3, then one per expert
+    g = np.full((B, E), -1e4)
+    g[:, 3] = 1e4
+    ent, bal, gate = o.router_stats(g, eps)
+    assert abs(ent - (-math.log(1.0 + eps))) <= 1e-20 and abs(bal - E) <= 1e-12
+    assert abs(gate - 1.0 / E) <= 1e-15
+    g = np.full((E, E), -1e4)
+    g[np.arange(E), np.arange(E)] = 1e4
+    assert abs(o.router_stats(g, eps)[1] - 1.0) <= 1e-14
+    # random batch against scipy's softmax and expit
+    rng = np.random.default_rng(21)
+    for E, B in ((7, 3), (172, 40), (224, 64)):
+        g = rng.standard_normal((B, E)) * 3.0
+        P = scipy.special.softmax(g, axis=1)
+        ent_ref = -np.sum(P * np.log(P + eps)) / B
+        bal_ref = E * np.sum(P.mean(axis=0) ** 2)
+        gate_ref = scipy.special.expit(g).mean()
+        ent, bal, gate = o.router_stats(g, eps)
+        assert abs(ent - ent_ref) <= 1e-12 * abs(ent_ref)
+        assert abs(bal - bal_ref) <= 1e-12 * bal_ref
+        assert abs(gate - gate_ref) <= 1e-13 * gate_ref
+    with pytest.raises(oracle.OracleError):
+        o.router_stats(np.array([[0.0, np.inf]]))
+
+
 def pin_special_p(o):
     rng = np.random.default_rng(16)
     E = 40
@@ -362,7 +396,8 @@ def pin_permutation_invariance(o):
 PINS = [pin_hand_selection, pin_hand_topk_lte, pin_hand_ffn, pin_logits_vs_matmul, pin_cum_vs_scipy_softmax,
         pin_bruteforce_min_prefix, pin_rank_restatement, pin_rule_relation, pin_special_p,
         pin_shift_invariance_and_huge_logits, pin_nonfinite, pin_activations, pin_dense_identity,
-        pin_masked_dense, pin_permutation_invariance, pin_topk_vs_lexsort, pin_lte_vs_expit]
+        pin_masked_dense, pin_permutation_invariance, pin_topk_vs_lexsort, pin_lte_vs_expit,
+        pin_router_stats]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -399,6 +434,11 @@ MUTANTS = {
     "topk_allows_zero": ("(p >= 1.0 ? (int)floor(p) : 1)", "(p >= 1.0 ? (int)floor(p) : 0)"),
     "lte_not_strict": ("ppo_sigmoid(order[r].g) > p)", "ppo_sigmoid(order[r].g) >= p)"),
     "lte_delta_le0_not_special": ("if (p <= 0.0 || ppo_sigmoid(order[r].g) > p)", "if (ppo_sigmoid(order[r].g) > p)"),
+    "stats_no_eps": ("ent -= pj * log(pj + eps);", "ent -= pj * log(pj);"),
+    "stats_ent_not_averaged": ("out[0] = ent / (double)T;", "out[0] = ent;"),
+    "stats_bal_not_squared": ("bal += f * f;", "bal += f;"),
+    "stats_bal_no_E": ("out[1] = (double)E * bal;", "out[1] = bal;"),
+    "stats_gate_raw_logit": ("gate += ppo_sigmoid(gt[j]);", "gate += gt[j];"),
     "lte_expert_order": ("idt[k++] = order[r].j;", "idt[k++] = order[E - 1 - r].j;"),
     "expert_block_offset": ("for (int n = e * de; n < (e + 1) * de; n++) {",
                             "for (int n = e * de + (de > 1); n < (e + 1) * de; n++) {"),
