@@ -44,6 +44,8 @@ def parse():
                     help="distinct token sets per layer (default 16 for decode batches, 1 for prefill)")
     ap.add_argument("--sweep", default="0.3,0.5,0.7,0.9,1.0", help="p values for the sweep ('' = none)")
     ap.add_argument("--sweep-steps", type=int, default=400)
+    ap.add_argument("--rules", default="topk:6,lte:0.995",
+                    help="other activation rules timed on the same kernels, rule:param ('' = none)")
     ap.add_argument("--no-flush", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--seed", type=int, default=0)
@@ -441,6 +443,25 @@ def main():
             for v in sweep.values():
                 v["speedup_vs_p1"] = v["tokens_per_s"] / dense["tokens_per_s"]
 
+    # ---- the other activation rules (top-k, LTE's threshold) on the same kernels
+    rules = {}
+    for item in [] if args.skip_extras else [v for v in args.rules.split(",") if v]:
+        rname, rp = item.split(":")
+        rpf = float(np.float32(float(rp)))
+        rdesc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act, "none" if rname == "lte" else "sigmoid", rname)
+        gs = capture_graphs(pp, rdesc, layers, rpf, B, args.pool, ws, stream)
+        tm = time_graphs(gs, args.sweep_steps, 5, flush, stream)
+        kk, un = selection_stats(pp, rdesc, layers, w, rpf, B, args.pool, ws)
+        sid = np.arange(args.sweep_steps) % args.pool
+        tb = sum(int((sid == i).sum()) * layer_bytes(w, B, int(un[i, l]))[0]
+                 for i in range(args.pool) for l in range(w.n_layers))
+        sec = sum(tm) / 1e3
+        rules[item] = {"tokens_per_s": B * args.sweep_steps / sec, "k_mean": float(kk.float().mean()),
+                       "total_gbs": tb / sec / 1e9, "frac_of_hbm_peak": tb / sec / 1e9 / hbm_peak}
+        del gs
+    if pp.pp_get_device_status(ws) != pp.PP_OK:
+        raise SystemExit("device status after the rule sweep: %s" % pp.status_name(pp.pp_get_device_status(ws)))
+
     if args.skip_extras:
         if rank == 0:
             print(json.dumps({"metric": METRIC, "value": value, "unit": "tokens/s", "ms_per_step": ms_per_step,
@@ -505,6 +526,26 @@ def main():
            "eager_value": replica_throughput(B * e2e_steps, timings["eager"], world, device)[0],
            "eager_path": "the same with the 32 pp_layer calls made eagerly every step"}
 
+    # ---- router statistics (L_ent, L_bal, L_gate) over a batch of 8192 tokens' logits
+    T_st = 8192
+    g_st = torch.randn((T_st, w.n_experts), device=device) * 3.0
+    ws_st = pp.alloc_workspace(desc, T_st)
+    out_st = torch.empty(3, dtype=torch.float64, device=device)
+    with torch.cuda.stream(stream):
+        for _ in range(5):
+            pp.pp_router_stats(desc, g_st, T_st, 1e-9, out_st, ws_st, stream=stream)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        n_st = 200
+        e0.record(stream)
+        for _ in range(n_st):
+            pp.pp_router_stats(desc, g_st, T_st, 1e-9, out_st, ws_st, stream=stream)
+        e1.record(stream)
+        stream.synchronize()
+    us_st = e0.elapsed_time(e1) * 1e3 / n_st
+    router_stats = {"tokens": T_st, "experts": w.n_experts, "us_per_call": us_st,
+                    "gbs": T_st * w.n_experts * 4 / (us_st * 1e-6) / 1e9,
+                    "note": "two launches (per-256-token parts, fixed-order final sum); logits L2-resident"}
+
     out = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
@@ -521,7 +562,7 @@ def main():
            "expert_bytes": {"gbs": expert_gbs, "frac_of_peak": expert_gbs / hbm_peak,
                             "frac_of_8tbs": expert_gbs / 8000.0, "k_mean": k_mean, "s_ffn": s_ffn},
            "hbm_gbs_total": tot_b / seconds / 1e9, "tflops": tot_f / seconds / 1e12,
-           "p_sweep": sweep, "warm_l2_tokens_per_s": warm_tok_s,
+           "p_sweep": sweep, "rules": rules, "router_stats": router_stats, "warm_l2_tokens_per_s": warm_tok_s,
            "e2e": e2e, "gpu_launches": launches * kernels_per_layer, "clocks": clocks}
     if rank == 0 and world == 1:
         try:

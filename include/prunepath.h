@@ -185,6 +185,20 @@ pp_status pp_layer_noalloc(const pp_desc *desc, const void *x, int T, const void
 pp_status pp_sparsity_stats(const int32_t *counts, int T, int n_experts, uint64_t *acc,
                             void *stream);
 
+/* Router statistics of a batch of B = T tokens (forward values of the router
+   terms of the training objective, reported as routing diagnostics):
+     out[0] = L_ent  = -(1/B) sum_t sum_j p_tj log(p_tj + eps)  (Sec. 3.2, Eq. entropy_loss)
+     out[1] = L_bal  = E sum_j ((1/B) sum_t p_tj)^2             (Sec. 3.2, Eq. load_balance_loss)
+     out[2] = L_gate = (1/(B E)) sum_t sum_j sigmoid(g_tj)       (Sec. 4.2.3, gate-magnitude term)
+   with p_tj the softmax of Eq. (softmax_prob).  logits [T][E] fp32 device
+   (e.g. the logits pp_route writes); out: 3 doubles, device, 8-byte aligned.
+   The softmax is max-shifted in fp32; the sums are fp64 in a fixed order
+   (deterministic).  T >= 1 (else PP_ERR_SHAPE); eps NaN is
+   PP_ERR_INVALID_ARG.  Uses the workspace of pp_workspace_size(desc, T).  A
+   non-finite logit records PP_ERR_NONFINITE and makes out[0] NaN. */
+pp_status pp_router_stats(const pp_desc *desc, const float *logits, int T, float eps, double *out, void *ws,
+                          size_t ws_bytes, void *stream);
+
 /* Synchronise `stream` and return the sticky device status of `ws`. */
 pp_status pp_get_device_status(void *ws, void *stream);
 

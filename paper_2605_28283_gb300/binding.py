@@ -57,6 +57,7 @@ EXPORTS = {
     "pp_layer": (_I, [_PD, _P, _I, _P, _P, _P, _P, _F, _PS, _P, _P, _Z, _P]),
     "pp_layer_noalloc": (_I, [_PD, _P, _I, _P, _P, _P, _P, _F, _PS, _P, _P, _P]),
     "pp_sparsity_stats": (_I, [_P, _I, _I, _P, _P]),
+    "pp_router_stats": (_I, [_PD, _P, _I, _F, _P, _P, _Z, _P]),
     "pp_get_device_status": (_I, [_P, _P]),
     "pp_debug_wait_timeout": (_I, [_P, _Z, _LL, _P]),
     "pp_status_string": (ctypes.c_char_p, [_I]),
@@ -196,6 +197,12 @@ def pp_layer_noalloc(desc, x, T, W_r, W_gate, W_up, W_down, p, sel_out, y, statu
 def pp_sparsity_stats(counts, T, n_experts, acc, stream=None):
     _check(load().pp_sparsity_stats(_ptr(counts), int(T), int(n_experts), _ptr(acc), _stream(stream)),
            "pp_sparsity_stats")
+
+
+def pp_router_stats(desc, logits, T, eps, out, ws, stream=None):
+    """L_ent, L_bal, L_gate of the logits [T][E] into out (3 float64, device)."""
+    _check(load().pp_router_stats(ctypes.byref(desc), _ptr(logits), int(T), float(eps), _ptr(out),
+                                  *_wsargs(ws), _stream(stream)), "pp_router_stats")
 
 
 def pp_get_device_status(ws, stream=None) -> int:

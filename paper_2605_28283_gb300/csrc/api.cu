@@ -52,7 +52,7 @@ bool use_grouped(const pp_desc& d, int T) { return d.dtype == PP_BF16 && T >= kG
 
 // Workspace layout for calls with up to T tokens.
 struct Layout {
-    size_t logits, ids, counts, gates, tlog, th;
+    size_t logits, ids, counts, gates, tlog, th, stats;
     // grouped path
     size_t part, bits, gexp, invpos, wcnt, blkcnt, blkbase, offsets, n_items, items, perm_token, perm_gate, H, Y,
         yacc, overflow;
@@ -75,6 +75,7 @@ Layout layout(const pp_desc& d, int T) {
     // tagged exchange words of the fused decode kernel (up to 8 tokens a launch)
     L.tlog = take(8 * E * 8);
     L.th = take(E * 8 * kDExpert * 8);
+    L.stats = take((size_t)router_stats_blocks((int)Tn) * (E + 2) * 8);
     if (use_grouped(d, T)) {
         const GroupedPlan g = grouped_plan(T, d.d_model, d.n_experts, 152);
         L.part = take((size_t)g.nsplit * Tn * E * 4);
@@ -476,6 +477,22 @@ pp_status pp_sparsity_stats(const int32_t* counts, int T, int n_experts, uint64_
     if (((uintptr_t)counts & 3u) || ((uintptr_t)acc & 7u)) return PP_ERR_ALIGN;
     PP_TRY(check_device());
     return cuda_status(stats_launch(counts, T, n_experts, acc, static_cast<cudaStream_t>(stream)));
+}
+
+pp_status pp_router_stats(const pp_desc* desc, const float* logits, int T, float eps, double* out, void* ws,
+                          size_t ws_bytes, void* stream) {
+    PP_TRY(check_desc(desc));
+    PP_TRY(check_T(desc, T));
+    if (T < 1) return PP_ERR_SHAPE;
+    if (std::isnan(eps) || !logits || !out) return PP_ERR_INVALID_ARG;
+    if (!aligned16(logits) || ((uintptr_t)out & 7u)) return PP_ERR_ALIGN;
+    PP_TRY(check_ws(desc, T, ws, ws_bytes));
+    PP_TRY(check_device());
+    char* b = static_cast<char*>(ws);
+    double* part = reinterpret_cast<double*>(b + layout(*desc, T).stats);
+    return cuda_status(router_stats_launch(logits, T, desc->n_experts, eps, part, out,
+                                           &reinterpret_cast<Control*>(b)->status,
+                                           static_cast<cudaStream_t>(stream)));
 }
 
 pp_status pp_get_device_status(void* ws, void* stream) {

@@ -489,9 +489,23 @@ __global__ void __launch_bounds__(1024) dispatch_small_kernel(const int32_t* __r
 // Persistent over work items.  NB = 128 (SwiGLU: gate rows then up rows) or
 // 64 (non-gated: up rows).  Two TMEM accumulators let the epilogue of one
 // item overlap the MMAs of the next.
+//
+// Warp roles: warp 0 streams the expert's weight tiles with 2-D TMA, warp 1
+// issues the MMAs, warps 2-5 run the epilogue, and warps 6-9 gather the
+// item's token rows: thread r copies row r of the A tile (128 bytes per
+// K chunk) with eight 16-byte cp.async into the 128-byte-swizzled layout the
+// TMA would write.  (A TMA gather4 moves 512 bytes per instruction and its
+// rate, about 14 GB/s per SM, bounded this kernel; cp.async keeps the L2
+// streaming.)  A gather thread keeps kGatherLag stages of copies in flight;
+// once a stage's copies are complete it fences them into the async proxy
+// and arrives on the stage's full barrier (129 arrivals: the weight TMA's
+// expect-tx arrival and the 128 gather threads).
+constexpr int kGuThreads = 320;
+constexpr int kGatherLag = 3;
+
 template <int NB>
-__global__ void __launch_bounds__(kTcThreads, 1)
-    gu_gemm_kernel(const __grid_constant__ CUtensorMap map_x1, const __grid_constant__ CUtensorMap map_wg,
+__global__ void __launch_bounds__(kGuThreads, 1)
+    gu_gemm_kernel(const __nv_bfloat16* __restrict__ x, int d, const __grid_constant__ CUtensorMap map_wg,
                    const __grid_constant__ CUtensorMap map_wu, const WorkItem* __restrict__ items,
                    const int* __restrict__ n_items_p, const int* __restrict__ perm_token,
                    const float* __restrict__ perm_gate, int nk, int act, __nv_bfloat16* H, unsigned* status,
@@ -499,6 +513,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
     pdl_launch_dependents();
     constexpr int kStages = NB == 128 ? 6 : 8;
+    static_assert(kGatherLag < kStages, "a gather thread must release a stage before it waits for it again");
     constexpr int kTileB = NB * 128;
     constexpr int kStage = kTileBytesA + kTileB;
     constexpr uint32_t kCols = 2 * NB;  // two accumulators
@@ -506,12 +521,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     __shared__ uint64_t full[kStages], empty[kStages], tfull[2], tempty[2];
     __shared__ uint32_t taddr_s;
-    __shared__ int rows_s[128];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int n_items = *n_items_p;
     if (threadIdx.x == 0) {
         for (int i = 0; i < kStages; i++) {
-            mbar_init(&full[i], 1);
+            mbar_init(&full[i], 1 + 128);
             mbar_init(&empty[i], 1);
         }
         for (int i = 0; i < 2; i++) {
@@ -530,28 +544,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const uint32_t tmem = taddr_s;
 
     if (warp == 0) {
-        int it = 0;
-        for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x) {
-            const WorkItem w = items[wi];
-            // the item's token rows (padding rows repeat the last token)
-            for (int i = lane; i < 128; i += 32) rows_s[i] = perm_token[w.a0 + min(i, w.cnt - 1)];
-            __syncwarp();
-            // only the item's live rows are gathered (lane g issues group g);
-            // padding rows keep stale data and only feed accumulator rows the
-            // epilogue never stores
-            const int ng = (w.cnt + 3) >> 2;
-            const int r0 = lane < ng ? rows_s[4 * lane] : 0, r1 = lane < ng ? rows_s[4 * lane + 1] : 0;
-            const int r2 = lane < ng ? rows_s[4 * lane + 2] : 0, r3 = lane < ng ? rows_s[4 * lane + 3] : 0;
-            for (int kc = 0; kc < nk; kc++, it++) {
-                const int s = it % kStages;
-                unsigned char* st = smem + (size_t)s * kStage;
-                if (lane == 0) {
+        if (lane == 0) {
+            int it = 0;
+            for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x) {
+                const WorkItem w = items[wi];
+                for (int kc = 0; kc < nk; kc++, it++) {
+                    const int s = it % kStages;
+                    unsigned char* st = smem + (size_t)s * kStage;
                     if (it >= kStages) mbar_wait(&empty[s], (uint32_t)((it / kStages) - 1) & 1u, status, lim);
-                    mbar_arrive_expect_tx(&full[s], (uint32_t)(ng * 512 + kTileB));
-                }
-                __syncwarp();
-                if (lane < ng) tma_gather4(st + lane * 512, &map_x1, kc * 64, r0, r1, r2, r3, &full[s]);
-                if (lane == 0) {
+                    mbar_arrive_expect_tx(&full[s], (uint32_t)kTileB);
                     if (NB == 128) {
                         tma_load_2d(st + kTileBytesA, &map_wg, kc * 64, w.e * 64, &full[s]);
                         tma_load_2d(st + kTileBytesA + 64 * 128, &map_wu, kc * 64, w.e * 64, &full[s]);
@@ -560,8 +561,42 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     }
                 }
             }
-            __syncwarp();
         }
+        __syncwarp();
+    } else if (warp >= 6) {
+        // token-row gather; rows past the item's count are not copied (their
+        // accumulator rows are never stored)
+        const int row = (warp - 6) * 32 + lane;
+        const uint32_t swz = (uint32_t)(row & 7);
+        int it = 0;
+        for (int wi = blockIdx.x; wi < n_items; wi += gridDim.x) {
+            const WorkItem w = items[wi];
+            const bool live = row < w.cnt;
+            const __nv_bfloat16* src = x + (size_t)(live ? perm_token[w.a0 + row] : 0) * d;
+            for (int kc = 0; kc < nk; kc++, it++) {
+                const int s = it % kStages;
+                if (lane == 0 && it >= kStages) mbar_wait(&empty[s], (uint32_t)((it / kStages) - 1) & 1u, status, lim);
+                __syncwarp();
+                unsigned char* dst = smem + (size_t)s * kStage + row * 128;
+                const int c0 = kc * 64;
+                if (live) {
+#pragma unroll
+                    for (int c = 0; c < 8; c++) {
+                        const bool in = c0 + c * 8 < d;  // d is a multiple of 8: chunks are whole
+                        cp_async_16(dst + (((uint32_t)c ^ swz) << 4), in ? src + c0 + c * 8 : src, in ? 16u : 0u);
+                    }
+                }
+                cp_async_commit();
+                if (it >= kGatherLag) {
+                    cp_async_wait<kGatherLag>();
+                    fence_proxy_async_smem();
+                    mbar_arrive(&full[(it - kGatherLag) % kStages]);
+                }
+            }
+        }
+        cp_async_wait<0>();
+        fence_proxy_async_smem();
+        for (int j = it > kGatherLag ? it - kGatherLag : 0; j < it; j++) mbar_arrive(&full[j % kStages]);
     } else if (warp == 1) {
         if (lane == 0) {
             constexpr uint32_t idesc = idesc_bf16_m128(NB);
@@ -1281,13 +1316,15 @@ cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
     } else if (gated) {
         const size_t smem = 6 * (size_t)(kTileBytesA + 128 * 128) + 1024;
         if ((e = set_smem(gu_gemm_kernel<128>, smem)) != cudaSuccess) return e;
-        PP_LAUNCH(gu_gemm_kernel<128>, dim3(grid), dim3(kTcThreads), smem, st, mx1, mwg, mwu, items, a.n_items,
-            a.perm_token, a.perm_gate, g.nk, a.act, a.H, a.status, a.timeout_ns);
+        PP_LAUNCH(gu_gemm_kernel<128>, dim3(grid), dim3(kGuThreads), smem, st,
+            reinterpret_cast<const __nv_bfloat16*>(a.x), a.d, mwg, mwu, items, a.n_items, a.perm_token, a.perm_gate,
+            g.nk, a.act, a.H, a.status, a.timeout_ns);
     } else {
         const size_t smem = 8 * (size_t)(kTileBytesA + 64 * 128) + 1024;
         if ((e = set_smem(gu_gemm_kernel<64>, smem)) != cudaSuccess) return e;
-        PP_LAUNCH(gu_gemm_kernel<64>, dim3(grid), dim3(kTcThreads), smem, st, mx1, mwg, mwu, items, a.n_items,
-            a.perm_token, a.perm_gate, g.nk, a.act, a.H, a.status, a.timeout_ns);
+        PP_LAUNCH(gu_gemm_kernel<64>, dim3(grid), dim3(kGuThreads), smem, st,
+            reinterpret_cast<const __nv_bfloat16*>(a.x), a.d, mwg, mwu, items, a.n_items, a.perm_token, a.perm_gate,
+            g.nk, a.act, a.H, a.status, a.timeout_ns);
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     // grouped down + scatter-add

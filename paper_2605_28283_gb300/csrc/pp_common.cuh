@@ -250,4 +250,10 @@ PP_DEVINL float warp_sum(float v) {
     return v;
 }
 
+PP_DEVINL float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(kFull, v, o));
+    return v;
+}
+
 }  // namespace pp

@@ -78,6 +78,9 @@ cudaError_t select_launch(const float* logits, int T, int E, float p, int rule, 
                           int32_t* ids, int32_t* counts, float* gates, unsigned* status,
                           cudaStream_t st);
 cudaError_t stats_launch(const int32_t* counts, int T, int E, uint64_t* acc, cudaStream_t st);
+int router_stats_blocks(int T);  // parts [blocks][E + 2] doubles of router_stats_launch
+cudaError_t router_stats_launch(const float* logits, int T, int E, float eps, double* part, double* out,
+                                unsigned* status, cudaStream_t st);
 cudaError_t wait_timeout_launch(unsigned* flag, unsigned* status, long long timeout_ns,
                                 cudaStream_t st);
 

@@ -115,6 +115,21 @@ PP_DEVINL void tma_gather4(void* dst, const CUtensorMap* map, int col, int r0, i
         : "memory");
 }
 
+// 16-byte cp.async global -> shared through L2 (not L1); src_bytes = 0
+// writes 16 zero bytes instead of reading.  Completion: cp_async_commit
+// closes a group, cp_async_wait<N> waits until at most N groups are pending.
+PP_DEVINL void cp_async_16(void* dst, const void* src, uint32_t src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src), "r"(src_bytes)
+                 : "memory");
+}
+
+PP_DEVINL void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+
+template <int N>
+PP_DEVINL void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
 // y[0..3] += v (fp32, one 16-byte vector reduction in L2)
 PP_DEVINL void red_add_v4(float* addr, float a, float b, float c, float d) {
     asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(addr), "f"(a), "f"(b), "f"(c), "f"(d)

@@ -154,6 +154,173 @@ cudaError_t stats_launch(const int32_t* counts, int T, int E, uint64_t* acc, cud
     return cudaGetLastError();
 }
 
+// ------------------------------------------------------ router statistics
+// Forward values of the router terms of the training objective (Sec. 3.2,
+// Eq. entropy_loss and Eq. load_balance_loss; L_gate of Sec. 4.2.3) over a
+// batch of logits [T][E].  Pass 1: CTA b takes tokens [64 b, 64 b + 64),
+// warp w eight of them, lane l the experts l + 32 s.  Per token the softmax
+// is max-shifted in fp32; a lane keeps the column sums of p over its warp's
+// tokens in fp32 and the entropy and sigmoid sums in fp64.  part[b] =
+// (column sums [E], sum p log(p + eps), sum sigmoid(g)), reduced over the
+// warps in a fixed order.  Pass 2 (one CTA of 1024 threads) sums the parts
+// in a fixed order with many loads in flight: the result is deterministic.
+constexpr int kStatTok = 64;
+constexpr int kStatFinal = 1024;
+
+__global__ void __launch_bounds__(256) router_stats_part_kernel(const float* __restrict__ logits, int T, int E,
+                                                                float eps, double* __restrict__ part,
+                                                                unsigned* status) {
+    __shared__ float colw[8][kMaxExperts];
+    __shared__ double entw[8], gatew[8];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int S = (E + 31) / 32;
+    float col[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    double ent = 0.0, gsum = 0.0;
+    const int per = kStatTok / 8;
+    const int tbeg = blockIdx.x * kStatTok + warp * per, tend = min(T, tbeg + per);
+    for (int t = tbeg; t < tend; t++) {
+        const float* row = logits + (size_t)t * E;
+        float g[8];
+        bool fin = true;
+        float m = -INFINITY;
+#pragma unroll
+        for (int s = 0; s < 8; s++) {
+            const int j = lane + 32 * s;
+            g[s] = (s < S && j < E) ? row[j] : -INFINITY;
+            if (s < S && j < E) fin = fin && isfinite(g[s]);
+            m = fmaxf(m, g[s]);
+        }
+        fin = __all_sync(kFull, fin);
+        m = warp_max(m);
+        float e[8], z = 0.0f;
+#pragma unroll
+        for (int s = 0; s < 8; s++) {
+            e[s] = (s < S && lane + 32 * s < E) ? expf(g[s] - m) : 0.0f;
+            z += e[s];
+        }
+        z = warp_sum(z);
+        float te = 0.0f, tg = 0.0f;
+#pragma unroll
+        for (int s = 0; s < 8; s++) {
+            if (s < S && lane + 32 * s < E) {
+                const float pj = e[s] / z;
+                col[s] += pj;
+                te += pj * logf(pj + eps);
+                tg += sigmoidf_(g[s]);
+            }
+        }
+        if (!fin) {
+            te = __int_as_float(0x7fc00000);  // NaN: the statistics of a batch with a non-finite logit
+            if (lane == 0) record_status(status, PP_ERR_NONFINITE);
+        }
+        ent += (double)te;
+        gsum += (double)tg;
+    }
+#pragma unroll
+    for (int s = 0; s < 8; s++)
+        if (s < S && lane + 32 * s < E) colw[warp][lane + 32 * s] = col[s];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        ent += __shfl_xor_sync(kFull, ent, o);
+        gsum += __shfl_xor_sync(kFull, gsum, o);
+    }
+    if (lane == 0) {
+        entw[warp] = ent;
+        gatew[warp] = gsum;
+    }
+    __syncthreads();
+    double* out = part + (size_t)blockIdx.x * (E + 2);
+    for (int j = threadIdx.x; j < E; j += blockDim.x) {
+        double c = 0.0;
+#pragma unroll
+        for (int w = 0; w < 8; w++) c += (double)colw[w][j];
+        out[j] = c;
+    }
+    if (threadIdx.x == 0) {
+        double a = 0.0, b = 0.0;
+#pragma unroll
+        for (int w = 0; w < 8; w++) {
+            a += entw[w];
+            b += gatew[w];
+        }
+        out[E] = a;
+        out[E + 1] = b;
+    }
+}
+
+// Sum of v over the CTA in a fixed order (warp shuffles, then warp 0 over
+// the warp sums); the result is valid in thread 0.
+PP_DEVINL double block_sum_fixed(double v, double* red) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+    __syncthreads();  // red may still be read by a previous call
+    if (lane == 0) red[warp] = v;
+    __syncthreads();
+    v = 0.0;
+    if (warp == 0) {
+        v = lane < nw ? red[lane] : 0.0;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+    }
+    return v;
+}
+
+__global__ void __launch_bounds__(kStatFinal) router_stats_final_kernel(const double* __restrict__ part, int nblk,
+                                                                        int T, int E, double* __restrict__ out) {
+    __shared__ double csum[4][kMaxExperts];
+    __shared__ double red[kStatFinal / 32];
+    // column sums: four threads per expert, each over a contiguous quarter of
+    // the parts with eight loads in flight
+    {
+        const int j = threadIdx.x >> 2, q = threadIdx.x & 3;
+        const int b0 = q * nblk / 4, b1 = (q + 1) * nblk / 4;
+        double c = 0.0;
+        if (j < E) {
+            int b = b0;
+            for (; b + 8 <= b1; b += 8) {
+                double v[8];
+#pragma unroll
+                for (int i = 0; i < 8; i++) v[i] = part[(size_t)(b + i) * (E + 2) + j];
+#pragma unroll
+                for (int i = 0; i < 8; i++) c += v[i];
+            }
+            for (; b < b1; b++) c += part[(size_t)b * (E + 2) + j];
+            csum[q][j] = c;
+        }
+    }
+    __syncthreads();
+    double sq = 0.0;
+    if (threadIdx.x < E) {
+        const int j = threadIdx.x;
+        const double f = (((csum[0][j] + csum[1][j]) + csum[2][j]) + csum[3][j]) / (double)T;  // (1/B) sum_t p_tj
+        sq = f * f;
+    }
+    double ent = 0.0, gate = 0.0;
+    for (int b = threadIdx.x; b < nblk; b += blockDim.x) {
+        ent += part[(size_t)b * (E + 2) + E];
+        gate += part[(size_t)b * (E + 2) + E + 1];
+    }
+    sq = block_sum_fixed(sq, red);
+    ent = block_sum_fixed(ent, red);
+    gate = block_sum_fixed(gate, red);
+    if (threadIdx.x == 0) {
+        out[0] = -ent / (double)T;
+        out[1] = (double)E * sq;
+        out[2] = gate / ((double)T * (double)E);
+    }
+}
+
+int router_stats_blocks(int T) { return (T + kStatTok - 1) / kStatTok; }
+
+cudaError_t router_stats_launch(const float* logits, int T, int E, float eps, double* part, double* out,
+                                unsigned* status, cudaStream_t st) {
+    const int nblk = router_stats_blocks(T);
+    router_stats_part_kernel<<<nblk, 256, 0, st>>>(logits, T, E, eps, part, status);
+    router_stats_final_kernel<<<1, kStatFinal, 0, st>>>(part, nblk, T, E, out);
+    return cudaGetLastError();
+}
+
 // ------------------------------------------------- bounded wait (test hook)
 // Waits for a flag that nothing sets; gives up after timeout_ns and records
 // PP_ERR_TIMEOUT.  Exercises the same bounded-wait path the kernels use.

@@ -117,3 +117,20 @@ def test_select_and_stats_validation(lib):
     assert L.pp_sparsity_stats(ctypes.c_void_p(A), 4, 300, ctypes.c_void_p(A), None) == pp.PP_ERR_INVALID_ARG
     assert L.pp_debug_wait_timeout(ctypes.c_void_p(A), 1 << 20, 0, None) == pp.PP_ERR_INVALID_ARG
     assert L.pp_workspace_init(ctypes.c_void_p(A + 8), 1 << 20, None) == pp.PP_ERR_WORKSPACE
+    ws = ctypes.c_void_p(A)
+    assert L.pp_router_stats(ctypes.byref(d), ctypes.c_void_p(A), 0, 1e-9, ctypes.c_void_p(A), ws, 1 << 30,
+                             None) == pp.PP_ERR_SHAPE
+    assert L.pp_router_stats(ctypes.byref(d), None, 4, 1e-9, ctypes.c_void_p(A), ws, 1 << 30,
+                             None) == pp.PP_ERR_INVALID_ARG
+    assert L.pp_router_stats(ctypes.byref(d), ctypes.c_void_p(A), 4, float("nan"), ctypes.c_void_p(A), ws,
+                             1 << 30, None) == pp.PP_ERR_INVALID_ARG
+    assert L.pp_router_stats(ctypes.byref(d), ctypes.c_void_p(A), 4, 1e-9, ctypes.c_void_p(A + 4), ws,
+                             1 << 30, None) == pp.PP_ERR_ALIGN
+    bad_rule = pp.make_desc(64, 16, "bf16", "swiglu")
+    bad_rule.rule = 4
+    assert L.pp_select(ctypes.byref(bad_rule), ctypes.c_void_p(A), 4, 0.5, ctypes.byref(sel),
+                       ctypes.c_void_p(A), 1 << 30, None) == pp.PP_ERR_INVALID_ARG
+    for rule in (pp.PP_SEL_TOPK, pp.PP_SEL_LTE):
+        d2 = pp.make_desc(64, 16, "bf16", "swiglu", rule=rule)
+        assert L.pp_select(ctypes.byref(d2), ctypes.c_void_p(A), 4, float("nan"), ctypes.byref(sel),
+                           ctypes.c_void_p(A), 1 << 30, None) == pp.PP_ERR_INVALID_ARG

@@ -25,12 +25,19 @@ def test_grouped_gelu(pp, T, p):
     layer_parity(pp, "gpt2m_gelu_bf16", T, p)
 
 
+@pytest.mark.parametrize("d,E,T", [(200, 9, 20), (1000, 40, 160)])
+def test_grouped_gelu_odd_shapes(pp, d, E, T):
+    """Non-gated FFN with d not a multiple of the 64-wide K chunk."""
+    layer_parity(pp, "gpt2m_gelu_bf16", T, 0.8, d=d, E=E)
+
+
 @pytest.mark.parametrize("rule,gate", [("paper", "sigmoid"), ("min_prefix", "none"), ("paper", "none")])
 def test_grouped_rules_gates(pp, rule, gate):
     layer_parity(pp, "llama2_7b_decode", 24, 0.6, rule, gate, d=1024, E=48)
 
 
-@pytest.mark.parametrize("d,E,T", [(128, 3, 5), (200, 33, 9), (512, 256, 33), (8192, 20, 6), (1024, 1, 7)])
+@pytest.mark.parametrize("d,E,T", [(128, 3, 5), (200, 33, 9), (512, 256, 33), (8192, 20, 6), (1024, 1, 7),
+                                   (200, 33, 150), (328, 7, 300)])
 def test_grouped_odd_shapes(pp, d, E, T):
     layer_parity(pp, "llama3_8b_batched", T, 0.8, d=d, E=E)
 

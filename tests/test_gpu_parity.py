@@ -346,6 +346,47 @@ def test_sparsity_stats(pp):
     np.testing.assert_array_equal(a[1:], 3 * np.bincount(counts, minlength=173))
 
 
+@pytest.mark.parametrize("T,E,std", [(1, 16, 3.0), (37, 172, 3.0), (256, 64, 1.0), (257, 224, 4.0),
+                                     (8192, 216, 3.0)])
+def test_router_stats(pp, T, E, std):
+    """L_ent, L_bal, L_gate against the oracle (fp32 softmax on the GPU)."""
+    import torch
+    logits = wl.host_logits(T, E, std=std, seed=T + E)
+    desc = pp.make_desc(64, E, "bf16", "swiglu")
+    ws = pp.alloc_workspace(desc, T)
+    out = torch.zeros(3, dtype=torch.float64, device="cuda")
+    for eps in (1e-9, 1e-2):
+        pp.pp_router_stats(desc, dev(logits), T, eps, out, ws)
+        torch.cuda.synchronize()
+        assert pp.pp_get_device_status(ws) == pp.PP_OK
+        ref = oracle.router_stats(logits.astype(np.float64), float(np.float32(eps)))
+        np.testing.assert_allclose(to_host(out), ref, rtol=2e-5, atol=1e-9)
+        again = torch.zeros_like(out)
+        pp.pp_router_stats(desc, dev(logits), T, eps, again, ws)
+        assert torch.equal(out, again)  # fixed reduction order
+
+
+def test_router_stats_closed_forms(pp):
+    import torch
+    E = 64
+    desc = pp.make_desc(64, E, "bf16", "swiglu")
+    ws = pp.alloc_workspace(desc, E)
+    out = torch.zeros(3, dtype=torch.float64, device="cuda")
+    g = np.full((E, E), -1e4, np.float32)
+    g[np.arange(E), np.arange(E)] = 1e4  # one expert per token, each expert once
+    pp.pp_router_stats(desc, dev(g), E, 1e-9, out, ws)
+    o = to_host(out)
+    assert abs(o[1] - 1.0) < 1e-6 and abs(o[0]) < 1e-6 and abs(o[2] - 1.0 / E) < 1e-7
+    g = np.zeros((E, E), np.float32)  # uniform routing
+    pp.pp_router_stats(desc, dev(g), E, 1e-9, out, ws)
+    o = to_host(out)
+    assert abs(o[0] - np.log(E)) < 1e-5 and abs(o[1] - 1.0) < 1e-6 and abs(o[2] - 0.5) < 1e-7
+    g[5, 7] = np.inf
+    pp.pp_router_stats(desc, dev(g), E, 1e-9, out, ws)
+    assert np.isnan(to_host(out)[0])
+    assert pp.pp_get_device_status(ws) == pp.PP_ERR_NONFINITE
+
+
 def test_bounded_wait_times_out(pp):
     """Failure detection: a wait on a flag nothing sets gives up and reports."""
     import torch
