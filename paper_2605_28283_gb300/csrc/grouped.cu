@@ -674,7 +674,8 @@ PP_DEVINL bool jt_first_overflow(const WorkItem& w, long long ycap) { return (lo
 // MMAs.
 __global__ void __launch_bounds__(kTcThreads, 1)
     down_gemm_kernel(const __grid_constant__ CUtensorMap map_h, const __grid_constant__ CUtensorMap map_wd,
-                     const WorkItem* __restrict__ items, const int* __restrict__ n_items_p,
+                     const __grid_constant__ CUtensorMap map_y, const WorkItem* __restrict__ items,
+                     const int* __restrict__ n_items_p,
                      const int* __restrict__ perm_token, int d, int njt, int nsub, __nv_bfloat16* Y, long long ycap,
                      float* yacc, int* overflow, unsigned* status, uint64_t lim) {
     pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
@@ -761,6 +762,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     } else {
         const int q = warp & 3;
         const int row = 32 * q + lane;
+        // this warp's staging area for bulk stores: four 64-column boxes of
+        // its 32 rows in the 128-byte swizzle (conflict-free row writes)
+        unsigned char* stage = smem + kTileBytesA + (size_t)kStages * kTileB + (size_t)q * 16384;
         int acc = 0;
         for (int v = blockIdx.x; v < n_tasks; v += gridDim.x) {
             const WorkItem w = items[v / nsub];
@@ -768,6 +772,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             slices(v, jt0, jt1);
             const bool live = row < w.cnt;
             const bool group_live = 32 * q < w.cnt;  // any live row in this warp's 32 rows
+            // all 32 rows live and inside Y: the group's rows go out as 2-D bulk stores
+            const bool group_full = 32 * q + 32 <= w.cnt && (long long)w.a0 + 32 * q + 32 <= ycap;
             const long long arow = (long long)w.a0 + row;
             const bool in_buf = live && arow < ycap;
             const int tok = live && !in_buf ? perm_token[arow] : -1;
@@ -779,8 +785,42 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 mbar_wait(&tfull[a], (uint32_t)(acc >> 1) & 1u, status, lim);
                 tc_fence_after();
                 const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(a * 256);
+                if (group_full) {
+                    // two halves of 128 columns; a half's two boxes are rewritten
+                    // only after the store that last used them has read them
 #pragma unroll 1
-                for (int c = 0; c < (group_live ? 256 : 0); c += 32) {
+                    for (int h = 0; h < 2; h++) {
+                        if (lane == 0) bulk_wait_read<1>();
+                        __syncwarp();
+#pragma unroll 1
+                        for (int c = 128 * h; c < 128 * h + 128; c += 32) {
+                            uint32_t r[32];
+                            tmem_ld32(base + (uint32_t)c, r);
+                            tmem_ld_wait();
+#pragma unroll
+                            for (int vv = 0; vv < 4; vv++) {
+                                const int j = (c >> 3) + vv;  // 16-byte chunk of the 256 columns
+                                const uint32_t off = (uint32_t)(j >> 3) * 4096u + (uint32_t)lane * 128u +
+                                                     ((((uint32_t)j & 7u) ^ ((uint32_t)lane & 7u)) << 4);
+                                *reinterpret_cast<uint4*>(stage + off) = make_uint4(
+                                    pack_bf16x2(__uint_as_float(r[8 * vv]), __uint_as_float(r[8 * vv + 1])),
+                                    pack_bf16x2(__uint_as_float(r[8 * vv + 2]), __uint_as_float(r[8 * vv + 3])),
+                                    pack_bf16x2(__uint_as_float(r[8 * vv + 4]), __uint_as_float(r[8 * vv + 5])),
+                                    pack_bf16x2(__uint_as_float(r[8 * vv + 6]), __uint_as_float(r[8 * vv + 7])));
+                            }
+                        }
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) {
+                            for (int b = 2 * h; b < 2 * h + 2; b++)
+                                if (jt * 256 + b * 64 < d)
+                                    tma_store_2d(&map_y, stage + b * 4096, jt * 256 + b * 64, w.a0 + 32 * q);
+                            bulk_commit();
+                        }
+                    }
+                }
+#pragma unroll 1
+                for (int c = 0; c < (group_live && !group_full ? 256 : 0); c += 32) {
                     uint32_t r[32];
                     tmem_ld32(base + (uint32_t)c, r);
                     tmem_ld_wait();
@@ -807,6 +847,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 if (lane == 0) mbar_arrive(&tempty[a]);
             }
         }
+        if (lane == 0) bulk_wait_all();  // the stores are done before the CTA's shared memory goes away
+        __syncwarp();
     }
     tc_fence_before();
     __syncthreads();
@@ -1344,14 +1386,17 @@ cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st) {
             a.perm_token, a.d, nrt, nsub, a.Y, g.ycap, a.yacc, a.overflow, a.status, a.timeout_ns);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     } else {
-        const size_t smem = (size_t)kTileBytesA + 4 * (size_t)256 * 128 + 1024;
+        // A tile, the 4-stage W_down ring, 4 x 16 KB store staging
+        const size_t smem = (size_t)kTileBytesA + 4 * (size_t)256 * 128 + 4 * (size_t)16384 + 1024;
+        CUtensorMap my;
+        if (!encode_2d(&my, a.Y, a.d, (uint64_t)g.ycap, 64, 32)) return cudaErrorInvalidValue;
         if ((e = set_smem(down_gemm_kernel, smem)) != cudaSuccess) return e;
         // up to 256 tokens: about one 128-row item per expert, fewer than the
         // SMs can share evenly, so each item's columns are cut into 4 tasks
         const int njt = (a.d + 255) / 256;
         const int nsub = a.T <= kSmallDispatchMaxT ? std::min(4, njt) : 1;
         const int grid6 = std::max(1, (int)std::min<long long>(sms, (long long)g.max_items * nsub));
-        PP_LAUNCH(down_gemm_kernel, dim3(grid6), dim3(kTcThreads), smem, st, mh, mwd, items, a.n_items, a.perm_token,
+        PP_LAUNCH(down_gemm_kernel, dim3(grid6), dim3(kTcThreads), smem, st, mh, mwd, my, items, a.n_items, a.perm_token,
             a.d, njt, nsub, a.Y, g.ycap, a.yacc, a.overflow, a.status, a.timeout_ns);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
