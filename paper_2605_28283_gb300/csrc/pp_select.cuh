@@ -193,7 +193,6 @@ struct CtaSelScratch {
     int ncand;
 };
 
-constexpr int kDecSelThreads = 256;  // the CTA selection runs on 8 warps
 
 PP_DEVINL uint32_t desc_key(float g) {
     unsigned u = __float_as_uint(g);
@@ -333,9 +332,11 @@ PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, bool want_rank,
         // summed over the candidates alone.  Below a bound of 20 * 2^-31
         // every expert is a candidate.
         filtered = true;
-        const float Bm = (1.0f - fmaxf(p, 0.0f)) * ((float)Z * (1.0f / 2147483648.0f)) / (float)E;
-        const float Lc = Bm >= 20.0f / 2147483648.0f ? logf(0.5f * Bm) : -INFINITY;
+        // the bound needs no rounding care (slack ln 2): fast log and divide
+        const float Bm = __fdividef((1.0f - fmaxf(p, 0.0f)) * ((float)Z * (1.0f / 2147483648.0f)), (float)E);
+        const float Lc = Bm >= 20.0f / 2147483648.0f ? __logf(0.5f * Bm) : -INFINITY;
         const bool cand = valid && (g - m) >= Lc;
+        const long long thr = prefix_threshold(p, Z);
         // compaction in arrival order through a warp-aggregated shared
         // counter; the key (D, index) carries the tie-break, and the slots
         // past the last candidate keep the padding written before the
@@ -351,15 +352,15 @@ PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, bool want_rank,
         }
         __syncthreads();
         const int nc = sc.ncand;
-        // nt threads per candidate (aligned lane groups), each summing a
-        // contiguous run of the candidates, four at a time
-        int nt = 16;
-        while (nt > 1 && nc * nt > kDecSelThreads) nt >>= 1;
-        const int q = j / nt, part = j % nt;
+        // nt = 2^lg threads per candidate (aligned lane groups), each summing
+        // a contiguous run of the candidates, four at a time
+        const int lg = nc <= 16 ? 4 : nc <= 32 ? 3 : nc <= 64 ? 2 : nc <= 128 ? 1 : 0;
+        const int nt = 1 << lg;
+        const int q = j >> lg, part = j & (nt - 1);
         unsigned long long a0 = 0ull, a1 = 0ull;
         if (q < nc) {
             const unsigned long long Kq = sK[q];
-            const int nv = (nc + 3) >> 2, per = (nv + nt - 1) / nt;
+            const int nv = (nc + 3) >> 2, per = (nv + nt - 1) >> lg;
             const int v1 = min(nv, (part + 1) * per);
             const ulonglong2* k2 = reinterpret_cast<const ulonglong2*>(sK);
             const uint4* u4p = reinterpret_cast<const uint4*>(sc.cu);
@@ -375,7 +376,6 @@ PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, bool want_rank,
         unsigned long long a = a0 + a1;
         for (int o = 1; o < nt; o <<= 1) a += __shfl_xor_sync(kFull, a, o);
         if (q < nc && part == 0) {
-            const long long thr = prefix_threshold(p, Z);
             const unsigned long long mass = rule == PP_SEL_PAPER ? a + sc.cu[q] : a;
             counted = a == 0ull || (thr >= 0 && mass <= (unsigned long long)thr);
             if (counted) sc.flag[(unsigned)sK[q] & 0xffu] = 1;
