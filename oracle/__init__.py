@@ -59,6 +59,8 @@ def load(path: str = None):
     lib.ppo_dense_ffn.argtypes = [_P, _I, _I, _I, _I, _I, _P, _P, _P, _I, _P]
     lib.ppo_router_stats.restype = _I
     lib.ppo_router_stats.argtypes = [_P, _I, _I, _D, _P]
+    lib.ppo_rmsnorm_residual.restype = _I
+    lib.ppo_rmsnorm_residual.argtypes = [_P, _P, _P, _I, _I, _I, _D, _P]
     lib.ppo_layer.restype = _I
     lib.ppo_layer.argtypes = [_P, _I, _I, _I, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _I, _P,
                               _P, _P, _P]
@@ -185,6 +187,24 @@ def router_stats(g, eps=1e-9):
     if s:
         raise OracleError(s, "ppo_router_stats")
     return float(out[0]), float(out[1]), float(out[2])
+
+
+def rmsnorm_residual(x_prev, y_prev=None, gamma=None, eps=1e-6):
+    """x = RMSNorm(x_prev + y_prev) * gamma per row, fp64.  Inputs share one
+    storage type; y_prev and gamma may be None."""
+    lib = load()
+    x_prev = _c(x_prev)
+    y_prev = None if y_prev is None else _c(y_prev)
+    gamma = None if gamma is None else _c(gamma)
+    T, d = x_prev.shape
+    dt = _dt(x_prev)
+    assert y_prev is None or (y_prev.shape == x_prev.shape and _dt(y_prev) == dt)
+    assert gamma is None or (gamma.shape == (d,) and _dt(gamma) == dt)
+    out = np.empty((T, d), np.float64)
+    s = lib.ppo_rmsnorm_residual(_ptr(x_prev), _ptr(y_prev), _ptr(gamma), dt, T, d, float(eps), _ptr(out))
+    if s:
+        raise OracleError(s, "ppo_rmsnorm_residual")
+    return out
 
 
 def layer(x, Wr, Wg, Wu, Wd, p, act_kind="swiglu", gate="sigmoid", rule="min_prefix"):

@@ -19,6 +19,8 @@
  *   Eq. (lte_hard_set)          A = {e : sigmoid(g_e) > delta}  (LTE's rule)
  * and the router statistics of the training objective (forward values):
  *   Eq. (entropy_loss), Eq. (load_balance_loss), L_gate (Sec. 4.2.3)          ppo_router_stats
+ * and, for chaining layers into a decode step, the residual + RMS
+ * normalisation x_{l+1} = RMSNorm(x_l + y_l)                                ppo_rmsnorm_residual
  * Every floating-point operation is done in double precision with plain
  * sequential loops; the inputs (fp32 or bf16) are widened exactly.
  *
@@ -420,4 +422,37 @@ int ppo_router_stats(const double *g, int T, int E, double eps, double *out)
     free(colsum);
     free(prob);
     return status;
+}
+
+/* ---- chained decode step ------------------------------------------------- */
+
+/*
+ * Input of the next layer of a stack of MoEfied FFN layers with a residual
+ * connection and RMS normalisation (the post-norm form x_{l+1} =
+ * RMSNorm(x_l + y_l)):
+ *   v = x_prev + y_prev                  (y_prev NULL: v = x_prev)
+ *   out = v / sqrt(mean(v^2) + eps) * gamma   (gamma NULL: unit weights)
+ * per token (row of d elements), in fp64.
+ */
+int ppo_rmsnorm_residual(const void *x_prev, const void *y_prev, const void *gamma, int dt, int T, int d,
+                         double eps, double *out)
+{
+    if (!dtype_ok(dt) || !x_prev || T < 0 || d <= 0 || isnan(eps))
+        return PPO_ERR_ARG;
+    for (int t = 0; t < T; t++) {
+        double ss = 0.0;
+        for (int i = 0; i < d; i++) {
+            double v = ld(x_prev, dt, (size_t)t * d + i);
+            if (y_prev)
+                v += ld(y_prev, dt, (size_t)t * d + i);
+            out[(size_t)t * d + i] = v;
+            ss += v * v;
+        }
+        const double r = 1.0 / sqrt(ss / (double)d + eps);
+        for (int i = 0; i < d; i++) {
+            const double g = gamma ? ld(gamma, dt, (size_t)i) : 1.0;
+            out[(size_t)t * d + i] *= r * g;
+        }
+    }
+    return PPO_OK;
 }

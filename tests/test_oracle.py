@@ -290,6 +290,31 @@ def pin_router_stats(o):
         o.router_stats(np.array([[0.0, np.inf]]))
 
 
+def pin_rmsnorm_residual(o):
+    """x_{l+1} = RMSNorm(x_l + y_l): closed forms, invariants and a numpy restatement."""
+    rng = np.random.default_rng(22)
+    # constant rows: c / sqrt(c^2 + eps)
+    x = np.full((2, 8), 3.0)
+    out = o.rmsnorm_residual(x, None, None, 0.25)
+    np.testing.assert_allclose(out, 3.0 / math.sqrt(9.25), rtol=1e-15)
+    # unit mean square at eps = 0; scale invariance; the residual is a plain sum
+    x = rng.standard_normal((5, 64))
+    y = rng.standard_normal((5, 64))
+    out = o.rmsnorm_residual(x, y, None, 0.0)
+    np.testing.assert_allclose((out ** 2).mean(axis=1), 1.0, rtol=1e-13)
+    np.testing.assert_allclose(o.rmsnorm_residual(7.5 * x, 7.5 * y, None, 0.0), out, rtol=1e-13)
+    np.testing.assert_allclose(o.rmsnorm_residual(x + y, None, None, 0.0), out, rtol=1e-13)
+    gamma = rng.uniform(0.5, 2.0, 64)
+    v = x + y
+    ref = v / np.sqrt((v ** 2).mean(axis=1, keepdims=True) + 1e-5) * gamma
+    np.testing.assert_allclose(o.rmsnorm_residual(x, y, gamma, 1e-5), ref, rtol=1e-13)
+    # bf16 inputs are widened exactly
+    xb, yb, gb = (wl.f32_to_bf16_bits(a.astype(np.float32)) for a in (x, y, gamma))
+    vb = widen(xb) + widen(yb)
+    refb = vb / np.sqrt((vb ** 2).mean(axis=1, keepdims=True) + 1e-6) * widen(gb)
+    np.testing.assert_allclose(o.rmsnorm_residual(xb, yb, gb, 1e-6), refb, rtol=1e-13)
+
+
 def pin_special_p(o):
     rng = np.random.default_rng(16)
     E = 40
@@ -397,7 +422,7 @@ PINS = [pin_hand_selection, pin_hand_topk_lte, pin_hand_ffn, pin_logits_vs_matmu
         pin_bruteforce_min_prefix, pin_rank_restatement, pin_rule_relation, pin_special_p,
         pin_shift_invariance_and_huge_logits, pin_nonfinite, pin_activations, pin_dense_identity,
         pin_masked_dense, pin_permutation_invariance, pin_topk_vs_lexsort, pin_lte_vs_expit,
-        pin_router_stats]
+        pin_router_stats, pin_rmsnorm_residual]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -439,6 +464,10 @@ MUTANTS = {
     "stats_bal_not_squared": ("bal += f * f;", "bal += f;"),
     "stats_bal_no_E": ("out[1] = (double)E * bal;", "out[1] = bal;"),
     "stats_gate_raw_logit": ("gate += ppo_sigmoid(gt[j]);", "gate += gt[j];"),
+    "norm_no_eps": ("const double r = 1.0 / sqrt(ss / (double)d + eps);", "const double r = 1.0 / sqrt(ss / (double)d);"),
+    "norm_sum_not_mean": ("const double r = 1.0 / sqrt(ss / (double)d + eps);", "const double r = 1.0 / sqrt(ss + eps);"),
+    "norm_no_residual": ("                v += ld(y_prev, dt, (size_t)t * d + i);", "                v += 0.0;"),
+    "norm_gamma_index": ("ld(gamma, dt, (size_t)i)", "ld(gamma, dt, (size_t)(d - 1 - i))"),
     "lte_expert_order": ("idt[k++] = order[r].j;", "idt[k++] = order[E - 1 - r].j;"),
     "expert_block_offset": ("for (int n = e * de; n < (e + 1) * de; n++) {",
                             "for (int n = e * de + (de > 1); n < (e + 1) * de; n++) {"),
