@@ -462,6 +462,37 @@ def main():
     if pp.pp_get_device_status(ws) != pp.PP_OK:
         raise SystemExit("device status after the rule sweep: %s" % pp.status_name(pp.pp_get_device_status(ws)))
 
+    # ---- chained decode step: layer l takes x_l = RMSNorm(x_{l-1} + y_{l-1}) (pp_layer_chained), so
+    # every layer reads the previous layer's output; one CUDA graph per pool entry
+    chained = None
+    if not args.skip_extras and B <= 4:
+        xs_c = [torch.empty((B, w.d_model), dtype=layers[0]["x"].dtype, device=device) for _ in range(w.n_layers)]
+        ys_c = [torch.empty_like(xs_c[0]) for _ in range(w.n_layers)]
+
+        def chain_step(i):
+            for l, L in enumerate(layers):
+                x_prev = L["x"][i] if l == 0 else xs_c[l - 1]
+                y_prev = None if l == 0 else ys_c[l - 1]
+                pp.pp_layer_chained(desc, x_prev, y_prev, None, 1e-6, B, L["Wr"], L["Wg"], L["Wu"], L["Wd"], pf,
+                                    None, xs_c[l], ys_c[l], ws, stream=stream)
+        gs = []
+        with torch.cuda.stream(stream):
+            for i in range(args.pool):
+                chain_step(i)
+            stream.synchronize()
+            for i in range(args.pool):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=stream):
+                    chain_step(i)
+                gs.append(g)
+        tm = time_graphs(gs, args.sweep_steps, 5, flush, stream)
+        if pp.pp_get_device_status(ws) != pp.PP_OK:
+            raise SystemExit("device status after the chained leg: %s" % pp.status_name(pp.pp_get_device_status(ws)))
+        chained = {"tokens_per_s": B * args.sweep_steps / (sum(tm) / 1e3), "ms_per_step": sum(tm) / args.sweep_steps,
+                   "what": "%d layers chained through pp_layer_chained: x_l = RMSNorm(x_(l-1) + y_(l-1)) formed "
+                           "in the fused decode kernel's prologue, layer 0 from the token input" % w.n_layers}
+        del gs
+
     if args.skip_extras:
         if rank == 0:
             print(json.dumps({"metric": METRIC, "value": value, "unit": "tokens/s", "ms_per_step": ms_per_step,
@@ -562,7 +593,7 @@ def main():
            "expert_bytes": {"gbs": expert_gbs, "frac_of_peak": expert_gbs / hbm_peak,
                             "frac_of_8tbs": expert_gbs / 8000.0, "k_mean": k_mean, "s_ffn": s_ffn},
            "hbm_gbs_total": tot_b / seconds / 1e9, "tflops": tot_f / seconds / 1e12,
-           "p_sweep": sweep, "rules": rules, "router_stats": router_stats, "warm_l2_tokens_per_s": warm_tok_s,
+           "p_sweep": sweep, "rules": rules, "chained": chained, "router_stats": router_stats, "warm_l2_tokens_per_s": warm_tok_s,
            "e2e": e2e, "gpu_launches": launches * kernels_per_layer, "clocks": clocks}
     if rank == 0 and world == 1:
         try:

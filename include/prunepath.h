@@ -156,6 +156,23 @@ pp_status pp_layer(const pp_desc *desc, const void *x, int T, const void *W_r, c
                    const void *W_up, const void *W_down, float p, const pp_selection *sel_out,
                    void *y, void *ws, size_t ws_bytes, void *stream);
 
+/* One layer of a chained decode step: the layer input is formed from the
+   previous layer's input and output,
+     x = RMSNorm(x_prev + y_prev) * gamma,   RMSNorm(v) = v / sqrt(mean(v^2) + eps)
+   per token (the post-norm residual connection x_{l+1} = RMSNorm(x_l + y_l)
+   that stacks the layers of the decode setting of Sec. 4.5), written to x,
+   and then y = pp_layer(x).  x_prev, y_prev, x, y are [T][d]; gamma is [d];
+   y_prev may be NULL (no residual term: the first layer) and gamma NULL
+   (unit weights).  The sum and the mean square are fp32; x is stored in the
+   desc dtype and the layer reads exactly that x.  For up to 4 bf16 / 8 fp32
+   tokens the fused decode kernel forms x in its prologue (one launch);
+   otherwise one more kernel runs first.  x and y must not overlap x_prev,
+   y_prev or each other (PP_ERR_INVALID_ARG); eps >= 0. */
+pp_status pp_layer_chained(const pp_desc *desc, const void *x_prev, const void *y_prev, const void *gamma,
+                           float eps, int T, const void *W_r, const void *W_gate, const void *W_up,
+                           const void *W_down, float p, const pp_selection *sel_out, void *x, void *y, void *ws,
+                           size_t ws_bytes, void *stream);
+
 /* pp_layer for callers that cannot allocate device memory where they run a
    layer -- a runtime that has given every byte to its own pool, a loop that
    must not block on an allocation's implicit synchronisation, a plug-in host
@@ -192,8 +209,8 @@ pp_status pp_sparsity_stats(const int32_t *counts, int T, int n_experts, uint64_
      out[2] = L_gate = (1/(B E)) sum_t sum_j sigmoid(g_tj)       (Sec. 4.2.3, gate-magnitude term)
    with p_tj the softmax of Eq. (softmax_prob).  logits [T][E] fp32 device
    (e.g. the logits pp_route writes); out: 3 doubles, device, 8-byte aligned.
-   The softmax is max-shifted in fp32; the sums are fp64 in a fixed order
-   (deterministic).  T >= 1 (else PP_ERR_SHAPE); eps NaN is
+   The softmax is max-shifted in fp32; the sums are fp32 in a fixed order,
+   pairwise across blocks of 64 tokens, combined in fp64 (deterministic).  T >= 1 (else PP_ERR_SHAPE); eps NaN is
    PP_ERR_INVALID_ARG.  Uses the workspace of pp_workspace_size(desc, T).  A
    non-finite logit records PP_ERR_NONFINITE and makes out[0] NaN. */
 pp_status pp_router_stats(const pp_desc *desc, const float *logits, int T, float eps, double *out, void *ws,

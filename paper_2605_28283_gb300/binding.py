@@ -55,6 +55,7 @@ EXPORTS = {
     "pp_select": (_I, [_PD, _P, _I, _F, _PS, _P, _Z, _P]),
     "pp_sparse_ffn": (_I, [_PD, _P, _I, _P, _P, _P, _PS, _P, _P, _Z, _P]),
     "pp_layer": (_I, [_PD, _P, _I, _P, _P, _P, _P, _F, _PS, _P, _P, _Z, _P]),
+    "pp_layer_chained": (_I, [_PD, _P, _P, _P, _F, _I, _P, _P, _P, _P, _F, _PS, _P, _P, _P, _Z, _P]),
     "pp_layer_noalloc": (_I, [_PD, _P, _I, _P, _P, _P, _P, _F, _PS, _P, _P, _P]),
     "pp_sparsity_stats": (_I, [_P, _I, _I, _P, _P]),
     "pp_router_stats": (_I, [_PD, _P, _I, _F, _P, _P, _Z, _P]),
@@ -184,6 +185,16 @@ def pp_layer(desc, x, T, W_r, W_gate, W_up, W_down, p, sel_out, y, ws, stream=No
     _check(load().pp_layer(ctypes.byref(desc), _ptr(x), int(T), _ptr(W_r), _ptr(W_gate), _ptr(W_up),
                            _ptr(W_down), float(p), None if s is None else ctypes.byref(s), _ptr(y),
                            *_wsargs(ws), _stream(stream)), "pp_layer")
+
+
+def pp_layer_chained(desc, x_prev, y_prev, gamma, eps, T, W_r, W_gate, W_up, W_down, p, sel_out, x, y, ws,
+                     stream=None):
+    """x = RMSNorm(x_prev + y_prev) * gamma, then y = pp_layer(x) (y_prev, gamma may be None)."""
+    s = None if sel_out is None else sel_out.c()
+    _check(load().pp_layer_chained(ctypes.byref(desc), _ptr(x_prev), _ptr(y_prev), _ptr(gamma), float(eps), int(T),
+                                   _ptr(W_r), _ptr(W_gate), _ptr(W_up), _ptr(W_down), float(p),
+                                   None if s is None else ctypes.byref(s), _ptr(x), _ptr(y), *_wsargs(ws),
+                                   _stream(stream)), "pp_layer_chained")
 
 
 def pp_layer_noalloc(desc, x, T, W_r, W_gate, W_up, W_down, p, sel_out, y, status_out=None, stream=None):

@@ -195,11 +195,19 @@ bool make_down_map(const pp_desc& d, const void* Wd, int R6, CUtensorMap* map) {
     return r == CUDA_SUCCESS;
 }
 
-DecodePlanIn plan_in(const pp_desc& d, int TS) {
+DecodePlanIn plan_in(const pp_desc& d, int TS, bool chain = false) {
     const DeviceInfo di = device_info();
     return DecodePlanIn{d.dtype, d.d_model, d.n_experts, TS, di.sms, d.act == PP_ACT_SWIGLU,
-                        di.smem_optin - kDecodeStaticSmemReserve};
+                        di.smem_optin - kDecodeStaticSmemReserve, chain};
 }
+
+// The chained step's extra inputs (pp_layer_chained); NULL for a plain layer.
+struct Chain {
+    const void* y_prev;
+    const void* gamma;
+    void* x_out;
+    float eps;
+};
 
 // Largest token count one fused decode launch takes for this shape (0: none).
 int decode_ts_limit(const pp_desc& d) {
@@ -257,13 +265,13 @@ GroupedArgs grouped_args(const pp_desc& d, int T, void* ws, const void* x, const
 // One launch of the fused decode kernel over tokens [t0, t0 + n).
 pp_status decode_call(const pp_desc& d, const void* x, int t0, int n, const void* Wr, const void* Wg,
                       const void* Wu, const void* Wd, float p, const pp_selection* sel, bool do_route,
-                      bool do_ffn, void* y, const Ws& w, cudaStream_t st) {
+                      bool do_ffn, void* y, const Ws& w, cudaStream_t st, const Chain* chain = nullptr) {
     const DeviceInfo di = device_info();
     int TS = 1;
     while (TS < n) TS <<= 1;
     if (TS > decode_max_ts(d.dtype)) return PP_ERR_SHAPE;
     DecodePlan plan;
-    if (!decode_plan(plan_in(d, TS), &plan)) return PP_ERR_SHAPE;
+    if (!decode_plan(plan_in(d, TS, chain != nullptr), &plan)) return PP_ERR_SHAPE;
     DecodeArgs a;
     std::memset(&a, 0, sizeof a);
     const size_t esz = d.dtype == PP_BF16 ? 2 : 4;
@@ -307,6 +315,15 @@ pp_status decode_call(const pp_desc& d, const void* x, int t0, int n, const void
     a.off_red6 = plan.off_red6;
     a.off_ring6 = plan.off_ring6;
     a.off_ring4 = plan.off_ring4;
+    a.off_chain = plan.off_chain;
+    if (chain) {
+        const size_t esz = d.dtype == PP_BF16 ? 2 : 4;
+        a.chain = 1;
+        a.y_prev = chain->y_prev ? static_cast<const char*>(chain->y_prev) + (size_t)t0 * d.d_model * esz : nullptr;
+        a.gamma = chain->gamma;
+        a.x_out = static_cast<char*>(chain->x_out) + (size_t)t0 * d.d_model * esz;
+        a.eps = chain->eps;
+    }
     return cuda_status(decode_launch(a, plan, d.dtype, TS, di.sms, st));
 }
 
@@ -472,6 +489,49 @@ pp_status pp_layer(const pp_desc* desc, const void* x, int T, const void* W_r, c
     return PP_OK;
 }
 
+pp_status pp_layer_chained(const pp_desc* desc, const void* x_prev, const void* y_prev, const void* gamma, float eps,
+                           int T, const void* W_r, const void* W_gate, const void* W_up, const void* W_down, float p,
+                           const pp_selection* sel_out, void* x, void* y, void* ws, size_t ws_bytes, void* stream) {
+    PP_TRY(check_desc(desc));
+    PP_TRY(check_T(desc, T));
+    if (std::isnan(p) || !(eps >= 0.0f)) return PP_ERR_INVALID_ARG;
+    if (sel_out) PP_TRY(check_sel(sel_out));
+    if (!x_prev || !x || !y || !W_r) return PP_ERR_INVALID_ARG;
+    if (!aligned16(x_prev) || !aligned16(x) || !aligned16(y) || !aligned16(W_r) || (y_prev && !aligned16(y_prev)) ||
+        (gamma && !aligned16(gamma)))
+        return PP_ERR_ALIGN;
+    // x and y are written while other CTAs may still read x_prev / y_prev
+    const size_t rows = (size_t)T * desc->d_model * (desc->dtype == PP_BF16 ? 2 : 4);
+    auto overlap = [rows](const void* a, const void* b) {
+        const char* pa = static_cast<const char*>(a);
+        const char* pb = static_cast<const char*>(b);
+        return a && b && pa < pb + rows && pb < pa + rows;
+    };
+    if (overlap(x, x_prev) || overlap(x, y_prev) || overlap(y, x_prev) || overlap(y, y_prev) || overlap(x, y))
+        return PP_ERR_INVALID_ARG;
+    PP_TRY(check_weights(desc, W_gate, W_up, W_down));
+    PP_TRY(check_ws(desc, T, ws, ws_bytes));
+    PP_TRY(check_device());
+    if (T == 0) return PP_OK;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const Ws w = ws_views(*desc, T, ws);
+    // fused: the decode kernel forms x in its prologue
+    if (!use_grouped(*desc, T)) {
+        const int ts = decode_ts_limit(*desc);
+        DecodePlan plan;
+        int TS = 1;
+        while (TS < T) TS <<= 1;
+        if (ts > 0 && T <= ts && decode_plan(plan_in(*desc, TS, true), &plan)) {
+            const float kp = rule_kernel_param(desc->rule, p, desc->n_experts);
+            const Chain c{y_prev, gamma, x, eps};
+            return decode_call(*desc, x_prev, 0, T, W_r, W_gate, W_up, W_down, kp, sel_out, true, true, y, w, st, &c);
+        }
+    }
+    // otherwise x first, then the layer on it
+    PP_TRY(cuda_status(rmsnorm_residual_launch(desc->dtype, x_prev, y_prev, gamma, eps, T, desc->d_model, x, st)));
+    return pp_layer(desc, x, T, W_r, W_gate, W_up, W_down, p, sel_out, y, ws, ws_bytes, stream);
+}
+
 pp_status pp_sparsity_stats(const int32_t* counts, int T, int n_experts, uint64_t* acc, void* stream) {
     if (!counts || !acc || T < 0 || n_experts < 1 || n_experts > kMaxExperts) return PP_ERR_INVALID_ARG;
     if (((uintptr_t)counts & 3u) || ((uintptr_t)acc & 7u)) return PP_ERR_ALIGN;
@@ -489,7 +549,7 @@ pp_status pp_router_stats(const pp_desc* desc, const float* logits, int T, float
     PP_TRY(check_ws(desc, T, ws, ws_bytes));
     PP_TRY(check_device());
     char* b = static_cast<char*>(ws);
-    double* part = reinterpret_cast<double*>(b + layout(*desc, T).stats);
+    float* part = reinterpret_cast<float*>(b + layout(*desc, T).stats);
     return cuda_status(router_stats_launch(logits, T, desc->n_experts, eps, part, out,
                                            &reinterpret_cast<Control*>(b)->status,
                                            static_cast<cudaStream_t>(stream)));

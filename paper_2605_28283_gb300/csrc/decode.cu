@@ -64,7 +64,9 @@ PP_DEVINL void load_given_selection(const DecodeArgs& a, float* gw, unsigned* ma
     }
 }
 
-template <typename TW, int TS, int RPL>
+// CHAIN: the chained step's prologue (a.chain) is compiled only into its own
+// instantiations, so that the plain layer's kernel carries no extra code.
+template <typename TW, int TS, int RPL, bool CHAIN>
 __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __grid_constant__ DecodeArgs a) {
     extern __shared__ __align__(1024) unsigned char smem[];
     using EL = Elem<TW>;
@@ -116,10 +118,15 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     }
     pdl_wait();
     pdl_launch_dependents();
+    TW* chain_y = reinterpret_cast<TW*>(ring4 + a.off_chain);
+    TW* chain_g = chain_y + (size_t)TS * d;
     if (tid == 0) {
         const uint32_t bytes = (uint32_t)(T * rowb);  // x -> shared memory (all T rows are contiguous)
-        mbar_arrive_expect_tx(&bars[kBarX], bytes);
+        const bool cy = CHAIN && a.y_prev, cg = CHAIN && a.gamma;
+        mbar_arrive_expect_tx(&bars[kBarX], bytes + (cy ? bytes : 0u) + (cg ? (uint32_t)rowb : 0u));
         bulk_g2s(xs, a.x, bytes, &bars[kBarX]);
+        if (cy) bulk_g2s(chain_y, a.y_prev, bytes, &bars[kBarX]);
+        if (cg) bulk_g2s(chain_g, a.gamma, (uint32_t)rowb, &bars[kBarX]);
         // this launch's tag: the CTA's launch count + 1 (its own word, last
         // written by this CTA in the previous launch, which has completed)
         const unsigned ep = a.epochs[b];
@@ -131,6 +138,48 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     mbar_wait(&bars[kBarX], 0, a.status, lim);
     __syncthreads();
     const unsigned tag = s_tag;
+
+    // chained step: the layer input is RMSNorm(x_prev + y_prev) * gamma, formed
+    // in place in shared memory by every CTA (CTA 0 also stores it)
+    if (CHAIN) {
+        for (int t = 0; t < T; t++) {
+            TW* xr = xs + (size_t)t * d;
+            const TW* yr = chain_y + (size_t)t * d;
+            float ss = 0.0f;
+            for (int c = tid; c < nchunk; c += kDecThreads) {
+                float xf[kEl], yf[kEl];
+                EL::unpack(reinterpret_cast<const uint4*>(xr)[c], xf);
+                if (a.y_prev) EL::unpack(reinterpret_cast<const uint4*>(yr)[c], yf);
+#pragma unroll
+                for (int q = 0; q < kEl; q++) {
+                    const float v = a.y_prev ? xf[q] + yf[q] : xf[q];
+                    ss = fmaf(v, v, ss);
+                }
+            }
+            ss = warp_sum(ss);
+            if (lane == 0) red[warp] = ss;
+            __syncthreads();
+            float tot = 0.0f;
+#pragma unroll
+            for (int w = 0; w < kWarps; w++) tot += red[w];
+            const float r = rsqrtf(tot / (float)d + a.eps);
+            for (int c = tid; c < nchunk; c += kDecThreads) {
+                float xf[kEl], yf[kEl], gf[kEl];
+                EL::unpack(reinterpret_cast<const uint4*>(xr)[c], xf);
+                if (a.y_prev) EL::unpack(reinterpret_cast<const uint4*>(yr)[c], yf);
+                if (a.gamma) EL::unpack(reinterpret_cast<const uint4*>(chain_g)[c], gf);
+#pragma unroll
+                for (int q = 0; q < kEl; q++) {
+                    const float v = a.y_prev ? xf[q] + yf[q] : xf[q];
+                    xf[q] = v * r * (a.gamma ? gf[q] : 1.0f);
+                }
+                const uint4 packed = EL::pack(xf);
+                reinterpret_cast<uint4*>(xr)[c] = packed;
+                if (b == 0) reinterpret_cast<uint4*>(static_cast<TW*>(a.x_out) + (size_t)t * d)[c] = packed;
+            }
+            __syncthreads();  // red is reused by the next token
+        }
+    }
 
     // ---------------------------------------------------------- phase 1
     if (a.do_route) {
@@ -547,6 +596,11 @@ bool decode_plan(const DecodePlanIn& in, DecodePlan* out) {
     p.off_ring4 = (uint32_t)off;
     if (off + stage4 > budget) return false;
     const size_t avail = budget - off;
+    // the ring also stages the router rows and, for a chained step, y_prev
+    // [TS][d] and gamma [d] (all read before phase 4 uses the ring)
+    p.off_chain = (uint32_t)align_up((size_t)rpc * in.d * esz, 128);
+    const size_t chain_end =
+        in.chain ? (size_t)p.off_chain + align_up((size_t)(TS + 1) * in.d * esz, 128) : (size_t)rpc * in.d * esz;
     const int ns4 = (int)std::min<size_t>(kMaxNS4, avail / stage4);
     // the ring also holds this CTA's router rows (phase 1) and, once phase 4
     // is done, the extra phase-6 slots plus at least one expert's h per warp
@@ -554,7 +608,7 @@ bool decode_plan(const DecodePlanIn& in, DecodePlan* out) {
     size_t ring4 = 0;
     int ext = kMaxSlots6 - p.ded6;
     for (; ext >= 0; ext--) {
-        ring4 = std::max({(size_t)ns4 * stage4, (size_t)rpc * in.d * esz,
+        ring4 = std::max({(size_t)ns4 * stage4, chain_end,
                           (size_t)ext * kWarps * stage6 + kWarps * hper});
         if (ring4 <= avail) break;
     }
@@ -571,7 +625,7 @@ bool decode_plan(const DecodePlanIn& in, DecodePlan* out) {
 
 template <typename TW, int TS, int RPL>
 static cudaError_t launch_one(const DecodeArgs& a, const DecodePlan& p, int grid, cudaStream_t st) {
-    auto kern = decode_layer_kernel<TW, TS, RPL>;
+    auto kern = a.chain ? decode_layer_kernel<TW, TS, RPL, true> : decode_layer_kernel<TW, TS, RPL, false>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg{};

@@ -212,6 +212,9 @@ struct Elem<float> {
         f[3] = __uint_as_float(v.w);
     }
     PP_DEVINL static void store(void* base, size_t i, float v) { reinterpret_cast<float*>(base)[i] = v; }
+    PP_DEVINL static uint4 pack(const float* f) {
+        return make_uint4(__float_as_uint(f[0]), __float_as_uint(f[1]), __float_as_uint(f[2]), __float_as_uint(f[3]));
+    }
 };
 
 template <>
@@ -229,6 +232,14 @@ struct Elem<__nv_bfloat16> {
     }
     PP_DEVINL static void store(void* base, size_t i, float v) {
         reinterpret_cast<__nv_bfloat16*>(base)[i] = __float2bfloat16_rn(v);
+    }
+    // round-to-nearest-even bf16 pairs, low half first
+    PP_DEVINL static uint32_t pair(float lo, float hi) {
+        const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+        return *reinterpret_cast<const uint32_t*>(&v);
+    }
+    PP_DEVINL static uint4 pack(const float* f) {
+        return make_uint4(pair(f[0], f[1]), pair(f[2], f[3]), pair(f[4], f[5]), pair(f[6], f[7]));
     }
 };
 

@@ -47,18 +47,29 @@ struct DecodeArgs {
     int do_route, do_ffn;
     int R6, NS4, ded6, slots6, hch;
     uint32_t off_x, off_gw, off_mask, off_ulist, off_red, off_red6, off_ring6, off_ring4;
+    // chained step: x = RMSNorm(x_prev + y_prev) * gamma computed in the
+    // prologue (a.x is then x_prev); y_prev and gamma staged in the phase-4
+    // ring at off_chain (free until phase 4), x written to x_out by CTA 0
+    int chain;
+    uint32_t off_chain;
+    const void* y_prev;
+    const void* gamma;
+    void* x_out;
+    float eps;
 };
 
 struct DecodePlanIn {
     int dtype, d, E, TS, grid;
     bool gated;
     size_t smem_limit;
+    bool chain = false;  // room for the chained step's y_prev and gamma
 };
 
 struct DecodePlan {
     int R6, RPL, NS4, ded6, slots6, hch, threads;
     size_t smem;
     uint32_t off_x, off_gw, off_mask, off_ulist, off_red, off_red6, off_ring6, off_ring4;
+    uint32_t off_chain;  // within the phase-4 ring: y_prev [TS][d] then gamma [d]
 };
 
 // Part of the per-block shared-memory limit left to the decode kernel's
@@ -78,8 +89,11 @@ cudaError_t select_launch(const float* logits, int T, int E, float p, int rule, 
                           int32_t* ids, int32_t* counts, float* gates, unsigned* status,
                           cudaStream_t st);
 cudaError_t stats_launch(const int32_t* counts, int T, int E, uint64_t* acc, cudaStream_t st);
-int router_stats_blocks(int T);  // parts [blocks][E + 2] doubles of router_stats_launch
-cudaError_t router_stats_launch(const float* logits, int T, int E, float eps, double* part, double* out,
+// x[t] = RMSNorm(x_prev[t] + y_prev[t]) * gamma (y_prev, gamma nullable), one CTA per token
+cudaError_t rmsnorm_residual_launch(int dtype, const void* x_prev, const void* y_prev, const void* gamma,
+                                    float eps, int T, int d, void* x, cudaStream_t st);
+int router_stats_blocks(int T);  // parts [blocks][E + 2] floats of router_stats_launch
+cudaError_t router_stats_launch(const float* logits, int T, int E, float eps, float* part, double* out,
                                 unsigned* status, cudaStream_t st);
 cudaError_t wait_timeout_launch(unsigned* flag, unsigned* status, long long timeout_ns,
                                 cudaStream_t st);

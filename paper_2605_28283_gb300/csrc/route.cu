@@ -159,23 +159,24 @@ cudaError_t stats_launch(const int32_t* counts, int T, int E, uint64_t* acc, cud
 // Eq. entropy_loss and Eq. load_balance_loss; L_gate of Sec. 4.2.3) over a
 // batch of logits [T][E].  Pass 1: CTA b takes tokens [64 b, 64 b + 64),
 // warp w eight of them, lane l the experts l + 32 s.  Per token the softmax
-// is max-shifted in fp32; a lane keeps the column sums of p over its warp's
-// tokens in fp32 and the entropy and sigmoid sums in fp64.  part[b] =
-// (column sums [E], sum p log(p + eps), sum sigmoid(g)), reduced over the
-// warps in a fixed order.  Pass 2 (one CTA of 1024 threads) sums the parts
-// in a fixed order with many loads in flight: the result is deterministic.
+// is max-shifted in fp32.  part[b] = (column sums of p [E], sum of
+// p log(p + eps), sum of sigmoid(g)) over the CTA's tokens, fp32, reduced over
+// the warps in a fixed order.  Pass 2 (one CTA of 1024 threads) adds the
+// parts pairwise in a fixed tree order and combines the totals in fp64: the
+// result is deterministic.  (This GPU's fp64 pipe is narrow, so fp64 is kept
+// to the final scalars.)
 constexpr int kStatTok = 64;
 constexpr int kStatFinal = 1024;
 
 __global__ void __launch_bounds__(256) router_stats_part_kernel(const float* __restrict__ logits, int T, int E,
-                                                                float eps, double* __restrict__ part,
+                                                                float eps, float* __restrict__ part,
                                                                 unsigned* status) {
     __shared__ float colw[8][kMaxExperts];
-    __shared__ double entw[8], gatew[8];
+    __shared__ float entw[8], gatew[8];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int S = (E + 31) / 32;
     float col[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-    double ent = 0.0, gsum = 0.0;
+    float ent = 0.0f, gsum = 0.0f;
     const int per = kStatTok / 8;
     const int tbeg = blockIdx.x * kStatTok + warp * per, tend = min(T, tbeg + per);
     for (int t = tbeg; t < tend; t++) {
@@ -213,31 +214,28 @@ __global__ void __launch_bounds__(256) router_stats_part_kernel(const float* __r
             te = __int_as_float(0x7fc00000);  // NaN: the statistics of a batch with a non-finite logit
             if (lane == 0) record_status(status, PP_ERR_NONFINITE);
         }
-        ent += (double)te;
-        gsum += (double)tg;
+        ent += te;
+        gsum += tg;
     }
 #pragma unroll
     for (int s = 0; s < 8; s++)
         if (s < S && lane + 32 * s < E) colw[warp][lane + 32 * s] = col[s];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        ent += __shfl_xor_sync(kFull, ent, o);
-        gsum += __shfl_xor_sync(kFull, gsum, o);
-    }
+    ent = warp_sum(ent);
+    gsum = warp_sum(gsum);
     if (lane == 0) {
         entw[warp] = ent;
         gatew[warp] = gsum;
     }
     __syncthreads();
-    double* out = part + (size_t)blockIdx.x * (E + 2);
+    float* out = part + (size_t)blockIdx.x * (E + 2);
     for (int j = threadIdx.x; j < E; j += blockDim.x) {
-        double c = 0.0;
+        float c = 0.0f;
 #pragma unroll
-        for (int w = 0; w < 8; w++) c += (double)colw[w][j];
+        for (int w = 0; w < 8; w++) c += colw[w][j];
         out[j] = c;
     }
     if (threadIdx.x == 0) {
-        double a = 0.0, b = 0.0;
+        float a = 0.0f, b = 0.0f;
 #pragma unroll
         for (int w = 0; w < 8; w++) {
             a += entw[w];
@@ -248,55 +246,49 @@ __global__ void __launch_bounds__(256) router_stats_part_kernel(const float* __r
     }
 }
 
-// Sum of v over the CTA in a fixed order (warp shuffles, then warp 0 over
-// the warp sums); the result is valid in thread 0.
-PP_DEVINL double block_sum_fixed(double v, double* red) {
+// Sum of v over the CTA in a fixed tree order (warp shuffles, then warp 0
+// over the warp sums); the result is valid in thread 0.
+PP_DEVINL float block_sum_fixed(float v, float* red) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+    v = warp_sum(v);
     __syncthreads();  // red may still be read by a previous call
     if (lane == 0) red[warp] = v;
     __syncthreads();
-    v = 0.0;
-    if (warp == 0) {
-        v = lane < nw ? red[lane] : 0.0;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
-    }
+    v = 0.0f;
+    if (warp == 0) v = warp_sum(lane < nw ? red[lane] : 0.0f);
     return v;
 }
 
-__global__ void __launch_bounds__(kStatFinal) router_stats_final_kernel(const double* __restrict__ part, int nblk,
+__global__ void __launch_bounds__(kStatFinal) router_stats_final_kernel(const float* __restrict__ part, int nblk,
                                                                         int T, int E, double* __restrict__ out) {
-    __shared__ double csum[4][kMaxExperts];
-    __shared__ double red[kStatFinal / 32];
+    __shared__ float csum[4][kMaxExperts];
+    __shared__ float red[kStatFinal / 32];
     // column sums: four threads per expert, each over a contiguous quarter of
-    // the parts with eight loads in flight
+    // the parts, eight loads in flight and a pairwise sum of each eight
     {
         const int j = threadIdx.x >> 2, q = threadIdx.x & 3;
         const int b0 = q * nblk / 4, b1 = (q + 1) * nblk / 4;
-        double c = 0.0;
+        float c = 0.0f;
         if (j < E) {
             int b = b0;
             for (; b + 8 <= b1; b += 8) {
-                double v[8];
+                float v[8];
 #pragma unroll
                 for (int i = 0; i < 8; i++) v[i] = part[(size_t)(b + i) * (E + 2) + j];
-#pragma unroll
-                for (int i = 0; i < 8; i++) c += v[i];
+                c += ((v[0] + v[1]) + (v[2] + v[3])) + ((v[4] + v[5]) + (v[6] + v[7]));
             }
             for (; b < b1; b++) c += part[(size_t)b * (E + 2) + j];
             csum[q][j] = c;
         }
     }
     __syncthreads();
-    double sq = 0.0;
+    float sq = 0.0f;
     if (threadIdx.x < E) {
         const int j = threadIdx.x;
-        const double f = (((csum[0][j] + csum[1][j]) + csum[2][j]) + csum[3][j]) / (double)T;  // (1/B) sum_t p_tj
+        const float f = ((csum[0][j] + csum[1][j]) + (csum[2][j] + csum[3][j])) / (float)T;  // (1/B) sum_t p_tj
         sq = f * f;
     }
-    double ent = 0.0, gate = 0.0;
+    float ent = 0.0f, gate = 0.0f;
     for (int b = threadIdx.x; b < nblk; b += blockDim.x) {
         ent += part[(size_t)b * (E + 2) + E];
         gate += part[(size_t)b * (E + 2) + E + 1];
@@ -305,20 +297,91 @@ __global__ void __launch_bounds__(kStatFinal) router_stats_final_kernel(const do
     ent = block_sum_fixed(ent, red);
     gate = block_sum_fixed(gate, red);
     if (threadIdx.x == 0) {
-        out[0] = -ent / (double)T;
-        out[1] = (double)E * sq;
-        out[2] = gate / ((double)T * (double)E);
+        out[0] = -(double)ent / (double)T;
+        out[1] = (double)E * (double)sq;
+        out[2] = (double)gate / ((double)T * (double)E);
     }
 }
 
 int router_stats_blocks(int T) { return (T + kStatTok - 1) / kStatTok; }
 
-cudaError_t router_stats_launch(const float* logits, int T, int E, float eps, double* part, double* out,
+cudaError_t router_stats_launch(const float* logits, int T, int E, float eps, float* part, double* out,
                                 unsigned* status, cudaStream_t st) {
     const int nblk = router_stats_blocks(T);
     router_stats_part_kernel<<<nblk, 256, 0, st>>>(logits, T, E, eps, part, status);
     router_stats_final_kernel<<<1, kStatFinal, 0, st>>>(part, nblk, T, E, out);
     return cudaGetLastError();
+}
+
+// ------------------------------------------------------- chained step
+// x[t] = RMSNorm(x_prev[t] + y_prev[t]) * gamma, one CTA of 256 threads per
+// token: the mean square in fp32 over 16-byte chunks, then the scaled rows
+// rounded to the storage type.  The fused decode kernel does the same in its
+// prologue; this kernel serves the grouped path and the token slices.
+template <typename TW>
+__global__ void __launch_bounds__(256) rmsnorm_residual_kernel(const TW* __restrict__ x_prev,
+                                                               const TW* __restrict__ y_prev,
+                                                               const TW* __restrict__ gamma, float eps, int d,
+                                                               TW* __restrict__ x) {
+    pdl_wait();  // x_prev / y_prev may be the previous kernel's output
+    pdl_launch_dependents();
+    using EL = Elem<TW>;
+    constexpr int kEl = EL::kPer16B;
+    __shared__ float red[8];
+    const int t = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nchunk = d / kEl;
+    const uint4* xr = reinterpret_cast<const uint4*>(x_prev + (size_t)t * d);
+    const uint4* yr = y_prev ? reinterpret_cast<const uint4*>(y_prev + (size_t)t * d) : nullptr;
+    float ss = 0.0f;
+    for (int c = threadIdx.x; c < nchunk; c += blockDim.x) {
+        float xf[kEl], yf[kEl];
+        EL::unpack(xr[c], xf);
+        if (yr) EL::unpack(yr[c], yf);
+#pragma unroll
+        for (int q = 0; q < kEl; q++) {
+            const float v = yr ? xf[q] + yf[q] : xf[q];
+            ss = fmaf(v, v, ss);
+        }
+    }
+    ss = warp_sum(ss);
+    if (lane == 0) red[warp] = ss;
+    __syncthreads();
+    float tot = 0.0f;
+#pragma unroll
+    for (int w = 0; w < 8; w++) tot += red[w];
+    const float r = rsqrtf(tot / (float)d + eps);
+    uint4* xo = reinterpret_cast<uint4*>(x + (size_t)t * d);
+    for (int c = threadIdx.x; c < nchunk; c += blockDim.x) {
+        float xf[kEl], yf[kEl], gf[kEl];
+        EL::unpack(xr[c], xf);
+        if (yr) EL::unpack(yr[c], yf);
+        if (gamma) EL::unpack(reinterpret_cast<const uint4*>(gamma)[c], gf);
+#pragma unroll
+        for (int q = 0; q < kEl; q++) xf[q] = (yr ? xf[q] + yf[q] : xf[q]) * r * (gamma ? gf[q] : 1.0f);
+        xo[c] = EL::pack(xf);
+    }
+}
+
+cudaError_t rmsnorm_residual_launch(int dtype, const void* x_prev, const void* y_prev, const void* gamma,
+                                    float eps, int T, int d, void* x, cudaStream_t st) {
+    if (T == 0) return cudaSuccess;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(T);
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (dtype == PP_BF16) {
+        using B = __nv_bfloat16;
+        return cudaLaunchKernelEx(&cfg, rmsnorm_residual_kernel<B>, static_cast<const B*>(x_prev),
+                                  static_cast<const B*>(y_prev), static_cast<const B*>(gamma), eps, d, static_cast<B*>(x));
+    }
+    return cudaLaunchKernelEx(&cfg, rmsnorm_residual_kernel<float>, static_cast<const float*>(x_prev),
+                              static_cast<const float*>(y_prev), static_cast<const float*>(gamma), eps, d,
+                              static_cast<float*>(x));
 }
 
 // ------------------------------------------------- bounded wait (test hook)
