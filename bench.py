@@ -577,6 +577,37 @@ def main():
                     "gbs": T_st * w.n_experts * 4 / (us_st * 1e-6) / 1e9,
                     "note": "two launches (per-256-token parts, fixed-order final sum); logits L2-resident"}
 
+    # ---- MoEfication repacking (Eq. permuted_weights) of one layer's weights by a random permutation
+    moefy_permute = None
+    if not args.skip_extras:
+        L0 = layers[0]
+        perm_d = torch.randperm(w.d_ff, device=device).to(torch.int32)
+        outs = [None if L0["Wg"] is None else torch.empty_like(L0["Wg"]), torch.empty_like(L0["Wu"]),
+                torch.empty_like(L0["Wd"])]
+        ws_mp = pp.alloc_workspace(desc, 0)
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                pp.pp_moefy_permute(desc, perm_d, L0["Wg"], L0["Wu"], L0["Wd"], *outs, ws_mp, stream=stream)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            n_mp = 20
+            e0.record(stream)
+            for _ in range(n_mp):
+                pp.pp_moefy_permute(desc, perm_d, L0["Wg"], L0["Wu"], L0["Wd"], *outs, ws_mp, stream=stream)
+            e1.record(stream)
+            stream.synchronize()
+        if pp.pp_get_device_status(ws_mp) != pp.PP_OK:
+            raise SystemExit("device status after the repacking leg: %s" % pp.status_name(pp.pp_get_device_status(ws_mp)))
+        pl = perm_d.long()
+        ok = torch.equal(outs[1][:64], L0["Wu"][pl[:64]]) and torch.equal(outs[2][:, :64], L0["Wd"][:, pl[:64]])
+        us_mp = e0.elapsed_time(e1) * 1e3 / n_mp
+        n_mat = 3 if L0["Wg"] is not None else 2
+        b_mp = 2 * n_mat * w.d_ff * w.d_model * L0["Wu"].element_size()
+        moefy_permute = {"us_per_call": us_mp, "bytes": b_mp, "gbs": b_mp / (us_mp * 1e-6) / 1e9,
+                         "frac_of_hbm_peak": b_mp / (us_mp * 1e-6) / 1e9 / hbm_peak, "spot_check": bool(ok),
+                         "what": "pp_moefy_permute of one layer (W_gate/W_up rows, W_down columns) by a random "
+                                 "permutation; bytes = read + write of the three matrices; 3 launches per call"}
+        del outs, ws_mp
+
     out = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
@@ -593,7 +624,8 @@ def main():
            "expert_bytes": {"gbs": expert_gbs, "frac_of_peak": expert_gbs / hbm_peak,
                             "frac_of_8tbs": expert_gbs / 8000.0, "k_mean": k_mean, "s_ffn": s_ffn},
            "hbm_gbs_total": tot_b / seconds / 1e9, "tflops": tot_f / seconds / 1e12,
-           "p_sweep": sweep, "rules": rules, "chained": chained, "router_stats": router_stats, "warm_l2_tokens_per_s": warm_tok_s,
+           "p_sweep": sweep, "rules": rules, "chained": chained, "router_stats": router_stats,
+           "moefy_permute": moefy_permute, "warm_l2_tokens_per_s": warm_tok_s,
            "e2e": e2e, "gpu_launches": launches * kernels_per_layer, "clocks": clocks}
     if rank == 0 and world == 1:
         try:

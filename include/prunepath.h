@@ -15,7 +15,8 @@
  * Conventions shared by every entry point
  *  - Every tensor pointer is a DEVICE pointer owned by the caller, row-major,
  *    contiguous and 16-byte aligned.  The library never allocates, frees or
- *    keeps a tensor pointer beyond the call.
+ *    keeps a tensor pointer beyond the call.  The one exception is the
+ *    offline host routine pp_moefy_cluster, whose pointers are host pointers.
  *  - Weight layout ("expert neurons stored contiguously"):
  *      W_r    [E][d]      row j is the routing vector of expert j
  *                         (the paper's W_r in R^{d x E}, stored transposed)
@@ -73,7 +74,9 @@ typedef enum pp_status {
     PP_ERR_CAPACITY = 8,    /* device: an internal buffer would overflow (sticky) */
     PP_ERR_NONFINITE = 9,   /* device: a router logit was NaN/Inf (sticky); the
                                token gets counts[t] = 0 and y[t] = 0              */
-    PP_ERR_UNSUPPORTED = 10 /* no device of compute capability 10.3 is current    */
+    PP_ERR_UNSUPPORTED = 10,/* no device of compute capability 10.3 is current    */
+    PP_ERR_HOST = 11        /* host memory or threads could not be obtained (the
+                               offline host routine pp_moefy_cluster)             */
 } pp_status;
 
 typedef enum pp_dtype { PP_F32 = 0, PP_BF16 = 1 } pp_dtype;
@@ -215,6 +218,54 @@ pp_status pp_sparsity_stats(const int32_t *counts, int T, int n_experts, uint64_
    non-finite logit records PP_ERR_NONFINITE and makes out[0] NaN. */
 pp_status pp_router_stats(const pp_desc *desc, const float *logits, int T, float eps, double *out, void *ws,
                           size_t ws_bytes, void *stream);
+
+/* MoEfication preprocessing, clustering (Sec. 2.2): group the d_ff
+   intermediate neurons of a dense FFN into E experts of d_e = 64 neurons by
+   balanced k-means over their input weights, and return the permutation Pi
+   that makes every expert a contiguous block (pp_moefy_permute applies it).
+   An OFFLINE HOST routine, run once per model before serving: W_gate, W_up,
+   init, perm, labels, iters and objective are HOST pointers; it runs on the
+   calling thread and a pool of host threads and touches no GPU.
+   - Features: neuron n's input weights -- row n of W_gate followed by row n
+     of W_up for PP_ACT_SWIGLU (W_gate required), row n of W_up otherwise
+     (W_gate ignored); W_gate, W_up are [d_ff][d] in desc->dtype, widened
+     exactly.
+   - Balanced k-means (the constrained k-means of Bradley, Bennett and
+     Demiriz, 2000, with every cluster holding exactly 64 neurons): the
+     centroids start at the features of neurons init[0..E) (distinct, in
+     [0, d_ff); the random choice is the caller's); each iteration assigns
+     the neurons to clusters with the least total squared Euclidean distance
+     under the equal-size constraint (solved exactly, fp64), then moves every
+     centroid to the mean of its members; it stops when an assignment repeats
+     the previous one, or after max_iter (>= 1) assignments.
+   - Outputs: perm [d_ff] int32 (new position j holds old neuron perm[j];
+     cluster e fills positions [64e, 64e + 64) in ascending old index);
+     labels [d_ff] int32, the cluster of each old neuron (may be NULL);
+     *iters = assignments made and *objective = the last assignment's sum of
+     squared distances (either may be NULL).
+   - Host memory: about d_ff * (f * 4 + E * 8) bytes, f = d or 2d.
+   Errors: PP_ERR_INVALID_ARG (NULL input or perm, bad init, max_iter < 1),
+   PP_ERR_SHAPE / PP_ERR_DTYPE as for every call, PP_ERR_HOST. */
+pp_status pp_moefy_cluster(const pp_desc *desc, const void *W_gate, const void *W_up, const int32_t *init,
+                           int max_iter, int32_t *perm, int32_t *labels, int *iters, double *objective);
+
+/* MoEfication preprocessing, repacking (Eq. permuted_weights:
+   W~_gate = W_gate Pi, W~_up = W_up Pi, W~_down = Pi^T W_down).  With the
+   neurons stored as rows of W_gate / W_up and columns of W_down:
+     W_gate_out[j][:] = W_gate[perm[j]][:],  W_up_out[j][:] = W_up[perm[j]][:],
+     W_down_out[:][j] = W_down[:][perm[j]]
+   so that expert e of the MoEfied FFN is the block of new neurons
+   [64e, 64e + 64) that every other call of this library reads.  Device
+   pointers: perm [d_ff] int32; weights in desc->dtype; W_gate / W_gate_out
+   are used only for PP_ACT_SWIGLU (required then).  No output may overlap an
+   input or another output (PP_ERR_INVALID_ARG).  Device-side check: an
+   entry of perm outside [0, d_ff), or repeated, records PP_ERR_INVALID_ARG
+   in the workspace status (pp_get_device_status); rows and columns for
+   out-of-range entries are written as zeros.  Workspace:
+   pp_workspace_size(desc, 0) bytes, initialised. */
+pp_status pp_moefy_permute(const pp_desc *desc, const int32_t *perm, const void *W_gate, const void *W_up,
+                           const void *W_down, void *W_gate_out, void *W_up_out, void *W_down_out, void *ws,
+                           size_t ws_bytes, void *stream);
 
 /* Synchronise `stream` and return the sticky device status of `ws`. */
 pp_status pp_get_device_status(void *ws, void *stream);

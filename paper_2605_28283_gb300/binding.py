@@ -13,7 +13,7 @@ from . import build as _build
 
 PP_OK, PP_ERR_INVALID_ARG, PP_ERR_SHAPE, PP_ERR_DTYPE, PP_ERR_ALIGN = 0, 1, 2, 3, 4
 PP_ERR_WORKSPACE, PP_ERR_CUDA, PP_ERR_TIMEOUT, PP_ERR_CAPACITY, PP_ERR_NONFINITE = 5, 6, 7, 8, 9
-PP_ERR_UNSUPPORTED = 10
+PP_ERR_UNSUPPORTED, PP_ERR_HOST = 10, 11
 PP_F32, PP_BF16 = 0, 1
 PP_ACT_RELU, PP_ACT_GELU_TANH, PP_ACT_SWIGLU = 0, 1, 2
 PP_GATE_SIGMOID, PP_GATE_NONE = 0, 1
@@ -59,6 +59,8 @@ EXPORTS = {
     "pp_layer_noalloc": (_I, [_PD, _P, _I, _P, _P, _P, _P, _F, _PS, _P, _P, _P]),
     "pp_sparsity_stats": (_I, [_P, _I, _I, _P, _P]),
     "pp_router_stats": (_I, [_PD, _P, _I, _F, _P, _P, _Z, _P]),
+    "pp_moefy_cluster": (_I, [_PD, _P, _P, _P, _I, _P, _P, _P, _P]),
+    "pp_moefy_permute": (_I, [_PD, _P, _P, _P, _P, _P, _P, _P, _P, _Z, _P]),
     "pp_get_device_status": (_I, [_P, _P]),
     "pp_debug_wait_timeout": (_I, [_P, _Z, _LL, _P]),
     "pp_status_string": (ctypes.c_char_p, [_I]),
@@ -214,6 +216,35 @@ def pp_router_stats(desc, logits, T, eps, out, ws, stream=None):
     """L_ent, L_bal, L_gate of the logits [T][E] into out (3 float64, device)."""
     _check(load().pp_router_stats(ctypes.byref(desc), _ptr(logits), int(T), float(eps), _ptr(out),
                                   *_wsargs(ws), _stream(stream)), "pp_router_stats")
+
+
+def _host(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def pp_moefy_cluster(desc, W_gate, W_up, init, max_iter=100):
+    """Balanced k-means of the neurons (host numpy arrays: float32, or uint16
+    bf16 bit patterns; init int32 [E]).  Returns (perm, labels, iters,
+    objective)."""
+    import numpy as np
+    W_up = np.ascontiguousarray(W_up)
+    W_gate = None if W_gate is None else np.ascontiguousarray(W_gate)
+    init = np.ascontiguousarray(init, dtype=np.int32)
+    perm = np.empty(desc.d_ff, np.int32)
+    labels = np.empty(desc.d_ff, np.int32)
+    iters = ctypes.c_int(0)
+    obj = ctypes.c_double(0.0)
+    _check(load().pp_moefy_cluster(ctypes.byref(desc), _host(W_gate), _host(W_up), _host(init), int(max_iter),
+                                   _host(perm), _host(labels), ctypes.byref(iters), ctypes.byref(obj)),
+           "pp_moefy_cluster")
+    return perm, labels, iters.value, obj.value
+
+
+def pp_moefy_permute(desc, perm, W_gate, W_up, W_down, W_gate_out, W_up_out, W_down_out, ws, stream=None):
+    """Eq. (permuted_weights) on the device: *_out = the weights with neuron j = old neuron perm[j]."""
+    _check(load().pp_moefy_permute(ctypes.byref(desc), _ptr(perm), _ptr(W_gate), _ptr(W_up), _ptr(W_down),
+                                   _ptr(W_gate_out), _ptr(W_up_out), _ptr(W_down_out), *_wsargs(ws),
+                                   _stream(stream)), "pp_moefy_permute")
 
 
 def pp_get_device_status(ws, stream=None) -> int:

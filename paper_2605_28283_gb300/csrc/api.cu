@@ -555,6 +555,54 @@ pp_status pp_router_stats(const pp_desc* desc, const float* logits, int T, float
                                            static_cast<cudaStream_t>(stream)));
 }
 
+pp_status pp_moefy_cluster(const pp_desc* desc, const void* W_gate, const void* W_up, const int32_t* init,
+                           int max_iter, int32_t* perm, int32_t* labels, int* iters, double* objective) {
+    PP_TRY(check_desc(desc));
+    const bool gated = desc->act == PP_ACT_SWIGLU;
+    if (!W_up || !init || !perm || (gated && !W_gate) || max_iter < 1) return PP_ERR_INVALID_ARG;
+    const int E = desc->n_experts, dff = desc->d_ff;
+    uint32_t seen[kMaxExperts * kDExpert / 32] = {};  // d_ff <= 256 * 64 bits
+    for (int h = 0; h < E; ++h) {
+        const int v = init[h];
+        if (v < 0 || v >= dff || (seen[v >> 5] >> (v & 31) & 1u)) return PP_ERR_INVALID_ARG;
+        seen[v >> 5] |= 1u << (v & 31);
+    }
+    return moefy_cluster_host(desc->dtype, gated ? W_gate : nullptr, W_up, dff, desc->d_model, E, init, max_iter,
+                              labels, perm, iters, objective);
+}
+
+pp_status pp_moefy_permute(const pp_desc* desc, const int32_t* perm, const void* W_gate, const void* W_up,
+                           const void* W_down, void* W_gate_out, void* W_up_out, void* W_down_out, void* ws,
+                           size_t ws_bytes, void* stream) {
+    PP_TRY(check_desc(desc));
+    const bool gated = desc->act == PP_ACT_SWIGLU;
+    if (!perm || !W_up_out || !W_down_out || (gated && !W_gate_out)) return PP_ERR_INVALID_ARG;
+    PP_TRY(check_weights(desc, gated ? W_gate : nullptr, W_up, W_down));
+    if (!aligned16(perm) || !aligned16(W_up_out) || !aligned16(W_down_out) || (gated && !aligned16(W_gate_out)))
+        return PP_ERR_ALIGN;
+    const size_t mat = (size_t)desc->d_ff * desc->d_model * (desc->dtype == PP_BF16 ? 2 : 4);
+    const char* in[3] = {static_cast<const char*>(gated ? W_gate : nullptr), static_cast<const char*>(W_up),
+                         static_cast<const char*>(W_down)};
+    const char* out[3] = {static_cast<const char*>(gated ? W_gate_out : nullptr),
+                          static_cast<const char*>(W_up_out), static_cast<const char*>(W_down_out)};
+    auto overlap = [mat](const char* a, const char* b) { return a && b && a < b + mat && b < a + mat; };
+    for (int i = 0; i < 3; ++i) {
+        for (int j = 0; j < 3; ++j) {
+            if (overlap(out[i], in[j])) return PP_ERR_INVALID_ARG;
+            if (j > i && overlap(out[i], out[j])) return PP_ERR_INVALID_ARG;
+        }
+        const char* pe = reinterpret_cast<const char*>(perm);
+        if (out[i] && out[i] < pe + (size_t)desc->d_ff * 4 && pe < out[i] + mat) return PP_ERR_INVALID_ARG;
+    }
+    PP_TRY(check_ws(desc, 0, ws, ws_bytes));
+    PP_TRY(check_device());
+    const DeviceInfo di = device_info();
+    return cuda_status(moefy_permute_launch(desc->dtype, perm, gated ? W_gate : nullptr, W_up, W_down,
+                                            gated ? W_gate_out : nullptr, W_up_out, W_down_out, desc->d_model,
+                                            desc->d_ff, di.sms, &static_cast<Control*>(ws)->status,
+                                            static_cast<cudaStream_t>(stream)));
+}
+
 pp_status pp_get_device_status(void* ws, void* stream) {
     if (!ws || ((uintptr_t)ws & 255u) != 0) return PP_ERR_WORKSPACE;
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -587,6 +635,7 @@ const char* pp_status_string(pp_status s) {
         case PP_ERR_CAPACITY: return "PP_ERR_CAPACITY";
         case PP_ERR_NONFINITE: return "PP_ERR_NONFINITE";
         case PP_ERR_UNSUPPORTED: return "PP_ERR_UNSUPPORTED";
+        case PP_ERR_HOST: return "PP_ERR_HOST";
     }
     return "PP_ERR_UNKNOWN";
 }

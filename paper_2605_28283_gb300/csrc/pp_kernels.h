@@ -146,6 +146,16 @@ GroupedPlan grouped_plan(int T, int d, int E, int sms);
 cudaError_t grouped_route(const GroupedArgs& a, cudaStream_t st);
 cudaError_t grouped_ffn(const GroupedArgs& a, int sms, cudaStream_t st);
 
+// ------------------------------------------------ MoEfication (Sec. 2.2)
+// Balanced k-means over the neurons' input weights (host, offline); shapes
+// and init already validated.  Returns PP_OK or PP_ERR_HOST.
+pp_status moefy_cluster_host(int dtype, const void* Wg, const void* Wu, int dff, int d, int E, const int32_t* init,
+                             int max_iter, int32_t* labels, int32_t* perm, int* iters, double* objective);
+// perm check + row gather (W_gate, W_up) + column gather (W_down); Wg NULL for non-gated FFNs
+cudaError_t moefy_permute_launch(int dtype, const int32_t* perm, const void* Wg, const void* Wu, const void* Wd,
+                                 void* Wg_out, void* Wu_out, void* Wd_out, int d, int dff, int sms, unsigned* status,
+                                 cudaStream_t st);
+
 // cuTensorMapEncodeTiled through the runtime's driver entry point (nullptr if unavailable)
 typedef CUresult (*TensorMapEncodeFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                       const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
