@@ -622,7 +622,8 @@ def main():
                             kernel="decode_layer_kernel" if B <= 4 else "pp_layer (grouped tcgen05 path)",
                             per="one pp_layer call (one layer)", launch_ms=per_launch_ms),
            "expert_bytes": {"gbs": expert_gbs, "frac_of_peak": expert_gbs / hbm_peak,
-                            "frac_of_8tbs": expert_gbs / 8000.0, "k_mean": k_mean, "s_ffn": s_ffn},
+                            "frac_of_8tbs": expert_gbs / 8000.0, "k_mean": k_mean, "k_min": int(ks.min()),
+                            "k_max": int(ks.max()), "s_ffn": s_ffn},
            "hbm_gbs_total": tot_b / seconds / 1e9, "tflops": tot_f / seconds / 1e12,
            "p_sweep": sweep, "rules": rules, "chained": chained, "router_stats": router_stats,
            "moefy_permute": moefy_permute, "warm_l2_tokens_per_s": warm_tok_s,
