@@ -140,3 +140,65 @@ def test_permute_argument_errors_on_the_host(lib):
     assert call(d=pp.make_desc(256, 4, "bf16", "swiglu", d_expert=16)) == pp.PP_ERR_SHAPE
     relu = pp.make_desc(256, 4, "bf16", "relu")
     assert call(d=relu, Wg=None, og=None) in (pp.PP_ERR_CUDA, pp.PP_ERR_UNSUPPORTED)
+
+
+# ------------------------------------------------ full-size optimality check
+def no_improving_exchange(D, labels, k, tol=1e-9):
+    """An equal-size assignment is optimal iff no cyclic exchange of neurons
+    between clusters lowers the cost, i.e. the graph on the clusters with
+    edge h -> h' = min over members j of h of D[j, h'] - D[j, h] has no
+    negative cycle (min-plus closure, Floyd-Warshall)."""
+    W = np.full((k, k), np.inf)
+    for h in range(k):
+        m = np.flatnonzero(labels == h)
+        W[h] = (D[m] - D[m, h][:, None]).min(axis=0)
+    np.fill_diagonal(W, 0.0)
+    for m in range(k):
+        W = np.minimum(W, W[:, m:m + 1] + W[m:m + 1, :])
+    return float(np.diag(W).min()) >= -tol
+
+
+def sq_dist(F32, C):
+    """||f - c||^2 for all pairs, fp64, in row blocks."""
+    out = np.empty((F32.shape[0], C.shape[0]))
+    cn = (C * C).sum(axis=1)
+    for i in range(0, F32.shape[0], 2048):
+        f = F32[i:i + 2048].astype(np.float64)
+        out[i:i + 2048] = (f * f).sum(axis=1)[:, None] - 2.0 * f @ C.T + cn[None, :]
+    return out
+
+
+@pytest.mark.parametrize("name", ["gpt2m_gelu_bf16", "llama2_7b_decode"])
+def test_full_size_assignments_are_optimal(lib, name):
+    """At the full layer shapes: the first assignment is optimal for the
+    initial centroids, and the converged labels are optimal for their own
+    cluster means (the fixed point of the iteration)."""
+    w = wl.WORKLOADS[name]
+    rng = np.random.default_rng(17)
+    mk = lambda: wl.f32_to_bf16_bits(rng.standard_normal((w.d_ff, w.d_model), dtype=np.float32) * np.float32(0.02))
+    Wg = mk() if w.gated else None
+    Wu = mk()
+    init = rng.choice(w.d_ff, size=w.n_experts, replace=False).astype(np.int32)
+    desc = pp.make_desc(w.d_model, w.n_experts, "bf16", w.act)
+    F32 = wl.bf16_bits_to_f32(Wu) if Wg is None else np.concatenate(
+        [wl.bf16_bits_to_f32(Wg), wl.bf16_bits_to_f32(Wu)], axis=1)
+    k = w.n_experts
+    # one assignment from the initial centroids
+    perm1, lab1, it1, obj1 = pp.pp_moefy_cluster(desc, Wg, Wu, init, 1)
+    assert it1 == 1 and np.array_equal(np.bincount(lab1, minlength=k), np.full(k, 64))
+    D1 = sq_dist(F32, F32[init].astype(np.float64))
+    assert no_improving_exchange(D1, lab1, k)
+    assert abs(D1[np.arange(w.d_ff), lab1].sum() - obj1) <= 1e-9 * obj1
+    # the check has teeth: swapping two neurons of different clusters leaves
+    # an improving exchange (the swap back)
+    i, j = 0, int(np.flatnonzero(lab1 != lab1[0])[0])
+    bad = lab1.copy()
+    bad[i], bad[j] = lab1[j], lab1[i]
+    assert not no_improving_exchange(D1, bad, k)
+    # the fixed point
+    perm, lab, it, obj = pp.pp_moefy_cluster(desc, Wg, Wu, init, 20)
+    assert 2 <= it < 20
+    C = np.stack([F32[lab == h].astype(np.float64).mean(axis=0) for h in range(k)])
+    D = sq_dist(F32, C)
+    assert no_improving_exchange(D, lab, k)
+    assert abs(D[np.arange(w.d_ff), lab].sum() - obj) <= 1e-9 * obj
