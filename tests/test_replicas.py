@@ -44,7 +44,7 @@ def _rank_main(rank, world, port, results):
 def test_two_replicas_report_all_tokens_over_the_slowest_rank():
     import torch.multiprocessing as mp
     pytest.importorskip("torch.distributed")
-    with mp.Manager() as m:
+    with mp.get_context("spawn").Manager() as m:  # no fork of this (multi-threaded) process
         results = m.dict()
         mp.spawn(_rank_main, args=(2, _free_port(), results), nprocs=2, join=True)
         res = dict(results)
