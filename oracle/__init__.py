@@ -61,6 +61,8 @@ def load(path: str = None):
     lib.ppo_router_stats.argtypes = [_P, _I, _I, _D, _P]
     lib.ppo_rmsnorm_residual.restype = _I
     lib.ppo_rmsnorm_residual.argtypes = [_P, _P, _P, _I, _I, _I, _D, _P]
+    lib.ppo_ffn_sparsity.restype = _I
+    lib.ppo_ffn_sparsity.argtypes = [_P, _I, _I, _I, _P, _P, _P]
     lib.ppo_layer.restype = _I
     lib.ppo_layer.argtypes = [_P, _I, _I, _I, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _I, _P,
                               _P, _P, _P]
@@ -205,6 +207,25 @@ def rmsnorm_residual(x_prev, y_prev=None, gamma=None, eps=1e-6):
     if s:
         raise OracleError(s, "ppo_rmsnorm_residual")
     return out
+
+
+def ffn_sparsity(counts, n_experts):
+    """Sec. 4.1: s_FFN of the activated-set sizes counts[L, N] (layer-major).
+    Returns (s_FFN, k_sum, hist) with hist[c] = #{(token, layer) : |A| = c},
+    c = 0..E."""
+    lib = load()
+    counts = np.ascontiguousarray(counts, dtype=np.int32)
+    if counts.ndim == 1:
+        counts = counts[None, :]
+    L, N = counts.shape
+    E = int(n_experts)
+    k_sum = np.zeros(1, np.uint64)
+    hist = np.zeros(E + 1, np.uint64)
+    s_ffn = np.zeros(1, np.float64)
+    s = lib.ppo_ffn_sparsity(_ptr(counts), N, L, E, _ptr(k_sum), _ptr(hist), _ptr(s_ffn))
+    if s:
+        raise OracleError(s, "ppo_ffn_sparsity")
+    return float(s_ffn[0]), int(k_sum[0]), hist.astype(np.int64)
 
 
 def layer(x, Wr, Wg, Wu, Wd, p, act_kind="swiglu", gate="sigmoid", rule="min_prefix"):

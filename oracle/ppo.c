@@ -21,6 +21,8 @@
  *   Eq. (entropy_loss), Eq. (load_balance_loss), L_gate (Sec. 4.2.3)          ppo_router_stats
  * and, for chaining layers into a decode step, the residual + RMS
  * normalisation x_{l+1} = RMSNorm(x_l + y_l)                                ppo_rmsnorm_residual
+ * and the efficiency metric of the experiments:
+ *   Sec. 4.1 (s_FFN)  s = 1 - (1/(N L E)) sum_i sum_l |A_l(x_i)|            ppo_ffn_sparsity
  * Every floating-point operation is done in double precision with plain
  * sequential loops; the inputs (fp32 or bf16) are widened exactly.
  *
@@ -454,5 +456,38 @@ int ppo_rmsnorm_residual(const void *x_prev, const void *y_prev, const void *gam
             out[(size_t)t * d + i] *= r * g;
         }
     }
+    return PPO_OK;
+}
+
+/* ---- FFN sparsity (Sec. 4.1) --------------------------------------------- */
+
+/*
+ * The average FFN sparsity of N tokens through L layers of E experts each:
+ *   s_FFN = 1 - (1 / (N L E)) sum_{i=1..N} sum_{l=1..L} |A_l(x_i)|
+ * where |A_l(x_i)| = counts[l * N + i], the number of experts activated for
+ * token i at layer l (0 <= count <= E; LTE's rule can activate none).
+ * Also returns the total sum of |A| (k_sum) and a histogram of the set sizes,
+ * hist[c] = #{(i, l) : |A_l(x_i)| = c} for c = 0..E (E + 1 entries).
+ * Returns PPO_ERR_ARG for N < 1, L < 1, E < 1 or a count outside [0, E].
+ */
+int ppo_ffn_sparsity(const int *counts, int N, int L, int E, unsigned long long *k_sum, unsigned long long *hist,
+                     double *s_ffn)
+{
+    if (!counts || N < 1 || L < 1 || E < 1)
+        return PPO_ERR_ARG;
+    for (int c = 0; c <= E; c++)
+        hist[c] = 0ull;
+    unsigned long long total = 0ull;
+    for (int i = 0; i < N; i++) {
+        for (int l = 0; l < L; l++) {
+            const int c = counts[(size_t)l * N + i];
+            if (c < 0 || c > E)
+                return PPO_ERR_ARG;
+            total += (unsigned long long)c;
+            hist[c] += 1ull;
+        }
+    }
+    *k_sum = total;
+    *s_ffn = 1.0 - (double)total / ((double)N * (double)L * (double)E);
     return PPO_OK;
 }

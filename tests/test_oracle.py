@@ -418,11 +418,38 @@ def pin_permutation_invariance(o):
     np.testing.assert_allclose(y, ref, rtol=1e-11, atol=1e-13)
 
 
+def pin_ffn_sparsity(o):
+    """Sec. 4.1 s_FFN: a hand-worked case, closed forms through the oracle's
+    own selection (p >= 1 activates all E, top-k exactly k, LTE at delta >= 1
+    none) and the histogram's two sums."""
+    case = json.load(open(GOLDEN))["ffn_sparsity"]
+    s, k_sum, hist = o.ffn_sparsity(np.array(case["counts"]), case["E"])
+    assert k_sum == case["k_sum"] and list(hist) == case["hist"]
+    assert abs(s - case["s_ffn_num"] / case["s_ffn_den"]) <= 1e-15
+    rng = np.random.default_rng(23)
+    E, N, L = 24, 7, 3
+    g = rng.standard_normal((L * N, E)) * 3.0
+    for p, rule, s_ref in ((1.0, "min_prefix", 0.0), (5.0, "topk", 1.0 - 5.0 / E), (1.0, "lte", 1.0),
+                           (0.0, "paper", 1.0 - 1.0 / E)):
+        counts = o.select(g, p, rule)[0].reshape(L, N)
+        s, k_sum, hist = o.ffn_sparsity(counts, E)
+        assert abs(s - s_ref) <= 1e-15, (p, rule, s)
+    # a mixed selection: the histogram counts every (token, layer) once and
+    # its first moment is the sum of the set sizes
+    counts = o.select(g, 0.7, "min_prefix")[0].reshape(L, N)
+    s, k_sum, hist = o.ffn_sparsity(counts, E)
+    assert hist.sum() == N * L and int((np.arange(E + 1) * hist).sum()) == k_sum
+    assert abs(s - (1.0 - k_sum / (N * L * E))) <= 1e-15
+    assert np.all(hist[np.bincount(counts.ravel(), minlength=E + 1) == 0] == 0)
+    with pytest.raises(oracle.OracleError):
+        o.ffn_sparsity(np.array([[E + 1]]), E)
+
+
 PINS = [pin_hand_selection, pin_hand_topk_lte, pin_hand_ffn, pin_logits_vs_matmul, pin_cum_vs_scipy_softmax,
         pin_bruteforce_min_prefix, pin_rank_restatement, pin_rule_relation, pin_special_p,
         pin_shift_invariance_and_huge_logits, pin_nonfinite, pin_activations, pin_dense_identity,
         pin_masked_dense, pin_permutation_invariance, pin_topk_vs_lexsort, pin_lte_vs_expit,
-        pin_router_stats, pin_rmsnorm_residual]
+        pin_router_stats, pin_rmsnorm_residual, pin_ffn_sparsity]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -469,6 +496,9 @@ MUTANTS = {
     "norm_no_residual": ("                v += ld(y_prev, dt, (size_t)t * d + i);", "                v += 0.0;"),
     "norm_gamma_index": ("ld(gamma, dt, (size_t)i)", "ld(gamma, dt, (size_t)(d - 1 - i))"),
     "lte_expert_order": ("idt[k++] = order[r].j;", "idt[k++] = order[E - 1 - r].j;"),
+    "sparsity_hist_off_by_one": ("hist[c] += 1ull;", "hist[c > 0 ? c - 1 : 0] += 1ull;"),
+    "sparsity_without_layers": ("((double)N * (double)L * (double)E)", "((double)N * (double)E)"),
+    "sparsity_not_complement": ("*s_ffn = 1.0 - (double)total", "*s_ffn = (double)total"),
     "expert_block_offset": ("for (int n = e * de; n < (e + 1) * de; n++) {",
                             "for (int n = e * de + (de > 1); n < (e + 1) * de; n++) {"),
 }
