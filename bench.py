@@ -41,7 +41,7 @@ def parse():
     ap.add_argument("--p", type=float, default=0.7)
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--pool", type=int, default=0,
-                    help="distinct token sets per layer (default 16 for decode batches, 1 for prefill)")
+                    help="distinct token sets per layer (default 64 for decode batches, 1 for prefill)")
     ap.add_argument("--sweep", default="0.3,0.5,0.7,0.9,1.0", help="p values for the sweep ('' = none)")
     ap.add_argument("--sweep-steps", type=int, default=400)
     ap.add_argument("--rules", default="topk:6,lte:0.995",
@@ -52,7 +52,16 @@ def parse():
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling runs)")
     ap.add_argument("--skip-extras", action="store_true",
                     help="only the headline timing (no warm/e2e/CPU legs); for profiler runs")
+    ap.add_argument("--configs", default="llama3_8b_batched:64:0.7,llama2_13b_prefill:8192:0.7:1,gpt2m_gelu_bf16:4:0.7",
+                    help="further workloads timed after the headline, workload:batch:p[:layers] ('' = none)")
+    ap.add_argument("--config-steps", type=int, default=300)
     return ap.parse_args()
+
+
+def default_pool(batch):
+    """Distinct token sets per layer that a step cycles through: 64 for
+    decode batches (expert choice changes every step), 1 for prefill."""
+    return 64 if batch <= 128 else 1
 
 
 def dist_env():
@@ -142,13 +151,13 @@ class ClockSampler:
 
 
 # -------------------------------------------------------------- workload
-def make_layers(w, args, device):
+def make_layers(w, B, pool, seed, device):
     import torch
     from paper_2605_28283_gb300 import workloads as wl
     layers = []
     for l in range(w.n_layers):
-        t = wl.device_layer(w, args.batch, args.seed, l, device, n_token_sets=args.pool)
-        t["y"] = torch.empty((args.batch, w.d_model), dtype=t["x"].dtype, device=device)
+        t = wl.device_layer(w, B, seed, l, device, n_token_sets=pool)
+        t["y"] = torch.empty((B, w.d_model), dtype=t["x"].dtype, device=device)
         layers.append(t)
     return layers
 
@@ -198,22 +207,27 @@ def time_graphs(graphs, steps, warmup, flush_buf, stream, profile_range=False):
 
 
 def selection_stats(pp, desc, layers, w, p, B, pool, ws):
-    """k per (pool entry, layer, token) via pp_route on the same inputs."""
+    """k per (pool entry, layer, token) and the union size |U| per (pool
+    entry, layer) via pp_route on the same inputs, and the s_FFN accumulators
+    (sum of k and its histogram, Sec. 4.1) from the library's own
+    pp_sparsity_stats over the same counts."""
     import numpy as np
     import torch
     ks = torch.empty((pool, len(layers), B), dtype=torch.int64)
     union = torch.empty((pool, len(layers)), dtype=torch.int64)
     sel = pp.Selection.empty(B, w.n_experts, "cuda", with_logits=False)
+    acc = torch.zeros(w.n_experts + 2, dtype=torch.int64, device="cuda")
     for i in range(pool):
         for l, L in enumerate(layers):
             pp.pp_route(desc, L["x"][i], B, L["Wr"], p, sel, ws)
+            pp.pp_sparsity_stats(sel.counts, B, w.n_experts, acc)
             c = sel.counts.cpu()
             ks[i, l] = c.long()
             ids = sel.ids.cpu().numpy()
             cn = c.numpy()
             mask = np.arange(ids.shape[1])[None, :] < cn[:, None]
             union[i, l] = len(np.unique(ids[mask]))
-    return ks, union
+    return ks, union, acc.cpu()
 
 
 def layer_bytes(w, B, n_union):
@@ -232,6 +246,12 @@ def layer_flops(w, B, k_sum):
     (token, activated expert), the gate/up and down products of a 64-wide block."""
     mats = 3 if w.gated else 2
     return 2.0 * B * w.n_experts * w.d_model + 2.0 * k_sum * mats * 64 * w.d_model
+
+
+def path_kind(w, B):
+    """Which kernels serve a pp_layer call: the fused decode kernel (bf16 up to
+    4 tokens, every fp32 call) or the grouped tensor-core path."""
+    return "decode" if (B <= 4 or w.dtype == "f32") else "grouped"
 
 
 def kernel_traffic(workload, p, B, kind="decode"):
@@ -265,78 +285,188 @@ def sources_sha(kind="decode"):
     return h.hexdigest()[:16]
 
 
+def roofline(w, B, p, bytes_per_launch, flops_per_launch, per_launch_ms):
+    """Roofline record of one pp_layer call: the bound is whichever of HBM
+    traffic and tensor work takes longer at the measured peaks; both
+    fractions are reported."""
+    hbm_peak, tc_peak, peak_kind = load_peaks()
+    sec = per_launch_ms / 1e3
+    hbm_gbs = bytes_per_launch / sec / 1e9
+    tflops = flops_per_launch / sec / 1e12
+    tensor_bound = flops_per_launch / (tc_peak * 1e12) > bytes_per_launch / (hbm_peak * 1e9)
+    kind = path_kind(w, B)
+    rec = {"bound": "tensor" if tensor_bound else "hbm",
+           "unit": "TFLOP/s" if tensor_bound else "GB/s",
+           "achieved": tflops if tensor_bound else hbm_gbs,
+           "peak": tc_peak if tensor_bound else hbm_peak,
+           "bytes_per_launch": bytes_per_launch, "flops_per_launch": flops_per_launch,
+           "hbm_frac": hbm_gbs / hbm_peak, "tensor_frac": tflops / tc_peak,
+           "traffic": kernel_traffic(w.name, p, B, kind), "peak_kind": peak_kind,
+           "kernel": "decode_layer_kernel" if kind == "decode" else "pp_layer (grouped tcgen05 path, all kernels)",
+           "per": "one pp_layer call (one layer)", "launch_ms": per_launch_ms}
+    rec["frac"] = rec["achieved"] / rec["peak"]
+    return rec
+
+
+def measure(pp, w, B, p, steps, warmup, pool, seed, device, stream, flush, world, rule="min_prefix",
+            gate="sigmoid", layers=None, profile_range=False, clocks=True):
+    """Times `steps` steps (one token set through every layer, one CUDA graph
+    per pool entry) and derives throughput, roofline and selection statistics
+    from the actual selections of the pool entries."""
+    import numpy as np
+    import torch
+    desc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act, gate, rule)
+    ws = pp.alloc_workspace(desc, B)
+    if layers is None:
+        layers = make_layers(w, B, pool, seed, device)
+    pf = float(np.float32(p))
+    graphs = capture_graphs(pp, desc, layers, pf, B, pool, ws, stream)
+    sampler = ClockSampler(torch.cuda.current_device()) if clocks else None
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.start()
+    times = time_graphs(graphs, steps, warmup, flush, stream, profile_range=profile_range)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clk = sampler.stop() if sampler else None
+    del graphs
+    value, slowest_s = replica_throughput(B * steps, sum(times) / 1e3, world, device)
+    status = pp.pp_get_device_status(ws)
+    if status != pp.PP_OK:
+        raise SystemExit("device status (%s B=%d p=%g): %s" % (w.name, B, p, pp.status_name(status)))
+    ks, union, acc = selection_stats(pp, desc, layers, w, pf, B, pool, ws)
+    step_ids = np.arange(steps) % pool
+    tot_b = exp_b = tot_f = 0.0
+    for i in range(pool):
+        n_i = int((step_ids == i).sum())
+        for l in range(w.n_layers):
+            a, e = layer_bytes(w, B, int(union[i, l]))
+            tot_b += n_i * a
+            exp_b += n_i * e
+            tot_f += n_i * layer_flops(w, B, int(ks[i, l].sum()))
+    seconds = sum(times) / 1e3
+    launches = steps * w.n_layers
+    per_launch_ms = sum(times) / launches   # step time / L: includes the in-graph launch gaps
+    hbm_peak = load_peaks()[0]
+    n_sel = pool * w.n_layers * B
+    k_sum = int(acc[0])
+    return {"tokens_per_s": value, "ms_per_step": slowest_s * 1e3 / steps, "steps": steps, "seconds": seconds,
+            "launches": launches, "per_launch_ms": per_launch_ms,
+            "roofline": roofline(w, B, p, tot_b / launches, tot_f / launches, per_launch_ms),
+            "expert_gbs": exp_b / seconds / 1e9, "total_gbs": tot_b / seconds / 1e9,
+            "frac_of_hbm_peak": tot_b / seconds / 1e9 / hbm_peak, "tflops": tot_f / seconds / 1e12,
+            "k_mean": k_sum / n_sel, "k_min": int(ks.min()), "k_max": int(ks.max()),
+            "union_mean": float(union.float().mean()),
+            "s_ffn": 1.0 - k_sum / (n_sel * w.n_experts),
+            "s_ffn_from": "pp_sparsity_stats over the pool's pp_route counts (%d token-layers)" % n_sel,
+            "clocks": clk, "ws": ws, "desc": desc, "layers": layers}
+
+
 # ------------------------------------------------------------ CPU oracle
-def run_oracle_sample(w, seconds, seed, host_layers=None, p=0.7, B=1):
-    """Times the oracle (as it stands) on a bounded sample of the workload:
-    whole-layer calls (logits, selection, sparse FFN) for B tokens, over a
-    few layers, repeated until `seconds` of CPU work; scaled to tokens/s of
-    the full L-layer model."""
+def cpu_env():
+    """Host cores: all of them, the ones this process may run on, and the
+    OpenMP threads the oracle's token loops may use."""
+    aff = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+    omp = int(os.environ.get("OMP_NUM_THREADS", aff))
+    return {"cpu_count": os.cpu_count(), "affinity_cores": aff, "omp_threads": omp}
+
+
+def oracle_sample_inputs(w, B, seed, n_layers=3, n_token_sets=8):
+    """Host inputs of the bounded oracle sample: n_layers distinct layers,
+    each with n_token_sets distinct token sets (the GPU arm likewise cycles
+    distinct token sets through distinct layers)."""
+    from paper_2605_28283_gb300 import workloads as wl
+    n_layers = max(1, min(n_layers, w.n_layers))
+    out = []
+    for l in range(n_layers):
+        L = wl.host_layer(w, B, seed=seed, layer=l)
+        toks = [L.x] + [wl.host_tokens(w, B, seed, l, stream=16 + j) for j in range(n_token_sets - 1)]
+        out.append((L, toks))
+    return out
+
+
+def oracle_calls(w, sample, p, B, seconds=None, calls=None):
+    """Runs single-layer oracle calls (logits, selection, sparse FFN), call i
+    on layer i mod n and on that layer's token set (i div n) mod m, until
+    `seconds` have passed or `calls` calls are done.  Returns (calls, s)."""
     import numpy as np
     import oracle
-    from paper_2605_28283_gb300 import workloads as wl
     oracle.load()
-    n_layers = 2 if host_layers is None else len(host_layers)
-    if host_layers is None:
-        host_layers = [wl.host_layer(w, B, seed=seed, layer=l) for l in range(n_layers)]
-    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
-    calls = 0
+    n, m = len(sample), len(sample[0][1])
+    pf = float(np.float32(p))
+    done = 0
     t0 = time.perf_counter()
     while True:
-        for L in host_layers:
-            oracle.layer(L.x, L.Wr, L.Wg, L.Wu, L.Wd, float(np.float32(p)), w.act, "sigmoid")
-            calls += 1
+        L, toks = sample[done % n]
+        oracle.layer(toks[(done // n) % m], L.Wr, L.Wg, L.Wu, L.Wd, pf, w.act, "sigmoid")
+        done += 1
         el = time.perf_counter() - t0
-        if el >= seconds:
-            break
+        if (seconds is not None and el >= seconds) or (calls is not None and done >= calls):
+            return done, el
+
+
+def oracle_record(w, B, calls, el, n_layers, n_sets, what):
+    env = cpu_env()
     per_layer = el / calls
-    tok_s = B / (per_layer * w.n_layers)
-    return {"value": tok_s, "unit": "tokens/s", "cores": min(threads, B) if B > 0 else 1, "kind": "oracle",
-            "sample": "%d calls of one layer x %d token(s) over %d distinct layers (%.1f s CPU); "
-                      "scaled to %d layers" % (calls, B, n_layers, el, w.n_layers)}
+    return {"value": B / (per_layer * w.n_layers), "unit": "tokens/s", "cores": max(1, min(env["omp_threads"], B)),
+            "kind": "oracle", **env,
+            "sample": "%s: %d single-layer calls x %d token(s), cycling %d distinct layers x %d distinct token "
+                      "sets (%.1f s CPU), scaled to %d layers" % (what, calls, B, n_layers, n_sets, el, w.n_layers)}
+
+
+def run_oracle_sample(w, seconds, seed, p=0.7, B=1):
+    """The cpu_baseline leg: the oracle as it stands on a bounded sample of
+    the workload, about `seconds` of CPU work."""
+    sample = oracle_sample_inputs(w, B, seed)
+    oracle_calls(w, sample, p, B, calls=1)   # load and first-touch
+    calls, el = oracle_calls(w, sample, p, B, seconds=seconds)
+    return oracle_record(w, B, calls, el, len(sample), len(sample[0][1]), "cpu_baseline leg")
+
+
+def config_dict(w, B, p, pool, world, no_flush):
+    return {"workload": w.name, "d_model": w.d_model, "d_ff": w.d_ff, "n_experts": w.n_experts,
+            "d_expert": 64, "layers": w.n_layers, "batch": B, "p": p, "act": w.act, "token_pool": pool,
+            "l2": "no flush (warm)" if no_flush else "flushed between steps (256 MiB write, untimed)",
+            "parallelism": "replicas" if world > 1 else "single GPU"}
 
 
 def run_reference(args):
+    """Reference arm: the CPU oracle as it stands, timed on the host cores on
+    the same workload, sampled exactly as the cpu_baseline leg samples it."""
     rank, world, _ = dist_env()
     from paper_2605_28283_gb300 import workloads as wl
     w = wl.WORKLOADS[args.workload]
     if rank != 0:
         return
-    # Each step is one bounded sample (a single layer call), scaled to the
-    # full model; the whole run stays within a few minutes.
-    import numpy as np
-    import oracle
-    oracle.load()
-    L = wl.host_layer(w, args.batch, seed=args.seed, layer=0)
-    p = float(np.float32(args.p))
-    for _ in range(max(1, min(args.warmup, 3))):
-        oracle.layer(L.x, L.Wr, L.Wg, L.Wu, L.Wd, p, w.act, "sigmoid")
-    steps = max(1, min(args.steps, 200))
-    t0 = time.perf_counter()
-    for _ in range(steps):
-        oracle.layer(L.x, L.Wr, L.Wg, L.Wu, L.Wd, p, w.act, "sigmoid")
-    el = time.perf_counter() - t0
-    per_step_model = el / steps * w.n_layers
-    value = args.batch / per_step_model
-    # the oracle's OpenMP loops run over tokens
-    cores = max(1, min(int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1)), args.batch))
+    B = args.batch
+    sample = oracle_sample_inputs(w, B, args.seed)
+    oracle_calls(w, sample, args.p, B, calls=max(1, min(args.warmup, 3)))
+    # each step is one single-layer call; the run is capped at about two minutes
+    steps, el = oracle_calls(w, sample, args.p, B, calls=max(1, min(args.steps, 5000)), seconds=120.0)
+    rec = oracle_record(w, B, steps, el, len(sample), len(sample[0][1]), "reference arm")
+    value = rec["value"]
     out = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus, "steps": steps,
-           "warmup": args.warmup, "ms_per_step": per_step_model * 1e3, "higher_is_better": True,
-           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-           "impl": "reference",
-           "config": {"workload": w.name, "d_model": w.d_model, "d_ff": w.d_ff, "n_experts": w.n_experts,
-                      "layers": w.n_layers, "batch": args.batch, "p": args.p},
-           "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-                            "sample": "%d single-layer calls (layer 0) x %d token(s), scaled to %d layers"
-                                      % (steps, args.batch, w.n_layers)},
+           "warmup": args.warmup, "ms_per_step": el / steps * w.n_layers * 1e3, "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+           "config": config_dict(w, B, args.p, args.pool, world, args.no_flush),
+           "cpu_baseline": rec,
            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out))
 
 
 # ------------------------------------------------------------------ main
+def public(m):
+    """A measurement record without its device objects."""
+    return {k: v for k, v in m.items() if k not in ("ws", "desc", "layers")}
+
+
 def main():
     args = parse()
     if args.pool <= 0:
-        args.pool = 16 if args.batch <= 128 else 1
+        args.pool = default_pool(args.batch)
     if args.impl == "reference":
         return run_reference(args)
     import numpy as np
@@ -357,10 +487,7 @@ def main():
         from dataclasses import replace
         w = replace(w, n_layers=args.layers)
     B = args.batch
-    desc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act)
     stream = torch.cuda.Stream()
-    ws = pp.alloc_workspace(desc, B)
-    layers = make_layers(w, args, device)
     flush = None if args.no_flush else torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=device)
     torch.cuda.synchronize()
 
@@ -371,101 +498,47 @@ def main():
 
     # ---- headline: p = args.p
     pf = float(np.float32(args.p))
-    graphs = capture_graphs(pp, desc, layers, pf, B, args.pool, ws, stream)
-    sampler = ClockSampler(local)
-    barrier()
-    sampler.start()
-    times = time_graphs(graphs, args.steps, args.warmup, flush, stream, profile_range=True)
-    barrier()
-    clocks = sampler.stop()
-    value, slowest_s = replica_throughput(B * args.steps, sum(times) / 1e3, world, device)
-    total_ms = slowest_s * 1e3
-    status = pp.pp_get_device_status(ws)
-    if status != pp.PP_OK:
-        raise SystemExit("device status: %s" % pp.status_name(status))
-    ms_per_step = total_ms / args.steps
+    head = measure(pp, w, B, args.p, args.steps, args.warmup, args.pool, args.seed, device, stream, flush, world,
+                   profile_range=True)
+    desc, ws, layers = head["desc"], head["ws"], head["layers"]
+    value, ms_per_step, roof = head["tokens_per_s"], head["ms_per_step"], head["roofline"]
+    head_rec = public(head)
+    kernels_per_layer = 1 if path_kind(w, B) == "decode" else 9
 
-    # bytes per step from the actual selections of the pool entries
-    ks, union = selection_stats(pp, desc, layers, w, pf, B, args.pool, ws)
-    step_ids = np.arange(args.steps) % args.pool
-    tot_b, exp_b, tot_f = 0.0, 0.0, 0.0
-    for i in range(args.pool):
-        n_i = int((step_ids == i).sum())
-        for l in range(w.n_layers):
-            a, e = layer_bytes(w, B, int(union[i, l]))
-            tot_b += n_i * a
-            exp_b += n_i * e
-            tot_f += n_i * layer_flops(w, B, int(ks[i, l].sum()))
-    seconds = sum(times) / 1e3
-    launches = args.steps * w.n_layers
-    # kernels of ours per layer call: the fused decode kernel (<= 4 bf16 / 8 fp32
-    # tokens), else router, selection, 4 dispatch kernels, gate/up, down, combine
-    kernels_per_layer = 1 if (B <= 4 or w.dtype == "f32") else 9
-    per_launch_ms = sum(times) / launches   # step time / L: includes the in-graph launch gaps
-    bytes_per_launch = tot_b / launches
-    flops_per_launch = tot_f / launches
-    hbm_peak, tc_peak, peak_kind = load_peaks()
-    # the bound is whichever of HBM traffic and tensor work takes longer at peak
-    tensor_bound = flops_per_launch / (tc_peak * 1e12) > bytes_per_launch / (hbm_peak * 1e9)
-    if tensor_bound:
-        achieved = flops_per_launch / (per_launch_ms / 1e3) / 1e12
-        peak = tc_peak
-        roof = {"bound": "tensor", "unit": "TFLOP/s", "flops_per_launch": flops_per_launch}
-    else:
-        achieved = bytes_per_launch / (per_launch_ms / 1e3) / 1e9
-        peak = hbm_peak
-        roof = {"bound": "hbm", "unit": "GB/s", "bytes_per_launch": bytes_per_launch}
-    expert_gbs = exp_b / seconds / 1e9
-    k_mean = float(ks.float().mean())
-    s_ffn = 1.0 - k_mean / w.n_experts
+    if args.skip_extras:
+        if rank == 0:
+            print(json.dumps({"metric": METRIC, "value": value, "unit": "tokens/s", "ms_per_step": ms_per_step,
+                              "workload": w.name, "layers": w.n_layers, "p": args.p, "batch": B,
+                              "launch_ms": head["per_launch_ms"], "bytes_per_launch": roof["bytes_per_launch"],
+                              "flops_per_launch": roof["flops_per_launch"], "roofline_bound": roof["bound"],
+                              "achieved": roof["achieved"], "peak": roof["peak"], "frac": roof["frac"],
+                              "sources_sha": sources_sha(path_kind(w, B))}))
+        return
 
     # ---- p sweep (same kernels), speedup vs dense p >= 1
     sweep = {}
-    if args.sweep:
-        for ps in [float(v) for v in args.sweep.split(",") if v]:
-            psf = float(np.float32(ps))
-            gs = capture_graphs(pp, desc, layers, psf, B, args.pool, ws, stream)
-            tm = time_graphs(gs, args.sweep_steps, 5, flush, stream)
-            kk, un = selection_stats(pp, desc, layers, w, psf, B, args.pool, ws)
-            sid = np.arange(args.sweep_steps) % args.pool
-            eb = sum(int((sid == i).sum()) * layer_bytes(w, B, int(un[i, l]))[1]
-                     for i in range(args.pool) for l in range(w.n_layers))
-            tb = sum(int((sid == i).sum()) * layer_bytes(w, B, int(un[i, l]))[0]
-                     for i in range(args.pool) for l in range(w.n_layers))
-            sec = sum(tm) / 1e3
-            sweep["%g" % ps] = {"tokens_per_s": B * args.sweep_steps / sec, "ms_per_step": sum(tm) / args.sweep_steps,
-                                "k_mean": float(kk.float().mean()), "s_ffn": 1 - float(kk.float().mean()) / w.n_experts,
-                                "expert_gbs": eb / sec / 1e9, "total_gbs": tb / sec / 1e9,
-                                "frac_of_hbm_peak": tb / sec / 1e9 / hbm_peak}
-            del gs
-        dense = sweep.get("1")
-        if dense:
-            for v in sweep.values():
-                v["speedup_vs_p1"] = v["tokens_per_s"] / dense["tokens_per_s"]
+    for ps in [float(v) for v in args.sweep.split(",") if v]:
+        m = measure(pp, w, B, ps, args.sweep_steps, 5, args.pool, args.seed, device, stream, flush, world,
+                    layers=layers, clocks=False)
+        sweep["%g" % ps] = {k: m[k] for k in ("tokens_per_s", "ms_per_step", "k_mean", "s_ffn", "expert_gbs",
+                                              "total_gbs", "frac_of_hbm_peak")}
+    dense = sweep.get("1")
+    if dense:
+        for v in sweep.values():
+            v["speedup_vs_p1"] = v["tokens_per_s"] / dense["tokens_per_s"]
 
     # ---- the other activation rules (top-k, LTE's threshold) on the same kernels
     rules = {}
-    for item in [] if args.skip_extras else [v for v in args.rules.split(",") if v]:
+    for item in [v for v in args.rules.split(",") if v]:
         rname, rp = item.split(":")
-        rpf = float(np.float32(float(rp)))
-        rdesc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act, "none" if rname == "lte" else "sigmoid", rname)
-        gs = capture_graphs(pp, rdesc, layers, rpf, B, args.pool, ws, stream)
-        tm = time_graphs(gs, args.sweep_steps, 5, flush, stream)
-        kk, un = selection_stats(pp, rdesc, layers, w, rpf, B, args.pool, ws)
-        sid = np.arange(args.sweep_steps) % args.pool
-        tb = sum(int((sid == i).sum()) * layer_bytes(w, B, int(un[i, l]))[0]
-                 for i in range(args.pool) for l in range(w.n_layers))
-        sec = sum(tm) / 1e3
-        rules[item] = {"tokens_per_s": B * args.sweep_steps / sec, "k_mean": float(kk.float().mean()),
-                       "total_gbs": tb / sec / 1e9, "frac_of_hbm_peak": tb / sec / 1e9 / hbm_peak}
-        del gs
-    if pp.pp_get_device_status(ws) != pp.PP_OK:
-        raise SystemExit("device status after the rule sweep: %s" % pp.status_name(pp.pp_get_device_status(ws)))
+        m = measure(pp, w, B, float(rp), args.sweep_steps, 5, args.pool, args.seed, device, stream, flush, world,
+                    rule=rname, gate="none" if rname == "lte" else "sigmoid", layers=layers, clocks=False)
+        rules[item] = {k: m[k] for k in ("tokens_per_s", "k_mean", "s_ffn", "total_gbs", "frac_of_hbm_peak")}
 
     # ---- chained decode step: layer l takes x_l = RMSNorm(x_{l-1} + y_{l-1}) (pp_layer_chained), so
     # every layer reads the previous layer's output; one CUDA graph per pool entry
     chained = None
-    if not args.skip_extras and B <= 4:
+    if B <= 4:
         xs_c = [torch.empty((B, w.d_model), dtype=layers[0]["x"].dtype, device=device) for _ in range(w.n_layers)]
         ys_c = [torch.empty_like(xs_c[0]) for _ in range(w.n_layers)]
 
@@ -493,24 +566,16 @@ def main():
                            "in the fused decode kernel's prologue, layer 0 from the token input" % w.n_layers}
         del gs
 
-    if args.skip_extras:
-        if rank == 0:
-            print(json.dumps({"metric": METRIC, "value": value, "unit": "tokens/s", "ms_per_step": ms_per_step,
-                              "workload": w.name, "layers": w.n_layers, "p": args.p, "batch": B,
-                              "launch_ms": per_launch_ms, "bytes_per_launch": bytes_per_launch,
-                              "flops_per_launch": flops_per_launch, "roofline_bound": roof["bound"],
-                              "achieved": achieved, "peak": peak, "frac": achieved / peak,
-                              "sources_sha": sources_sha("decode" if B <= 4 or w.dtype == "f32" else "grouped")}))
-        return
-
     # ---- warm-L2 number (no flush), for context
+    graphs = capture_graphs(pp, desc, layers, pf, B, args.pool, ws, stream)
     warm = time_graphs(graphs, min(args.steps, 500), 5, None, stream)
     warm_tok_s = B * len(warm) / (sum(warm) / 1e3)
+    del graphs
 
     # ---- end to end through the public API with host buffers.  Every step
-    # copies the 32 layer inputs from pinned host memory in one transfer,
-    # replays a CUDA graph of the 32 pp_layer calls (captured once through
-    # the binding) and reads the 32 outputs back; the host waits for them.
+    # copies the L layer inputs from pinned host memory in one transfer,
+    # replays a CUDA graph of the L pp_layer calls (captured once through
+    # the binding) and reads the L outputs back; the host waits for them.
     esz = 2 if w.dtype == "bf16" else 4
     dt = layers[0]["x"].dtype
     npool = min(args.pool, 16)
@@ -548,14 +613,15 @@ def main():
                     y_host.copy_(y_dev, non_blocking=True)
                     stream.synchronize()
                 timings[mode] = time.perf_counter() - t0
+    del g_e2e
     e2e = {"value": replica_throughput(B * e2e_steps, timings["graph"], world, device)[0],
            "unit": "tokens/s", "h2d_bytes_per_step": w.n_layers * B * w.d_model * esz,
            "d2h_bytes_per_step": w.n_layers * B * w.d_model * esz,
-           "path": "pp_layer via the ctypes binding, 32 calls captured once in a CUDA graph; per step one "
-                   "pinned H2D copy of the 32 layer inputs, graph replay, one D2H copy of the 32 outputs, "
-                   "host synchronisation",
+           "path": "pp_layer via the ctypes binding, %d calls captured once in a CUDA graph; per step one "
+                   "pinned H2D copy of the %d layer inputs, graph replay, one D2H copy of the %d outputs, "
+                   "host synchronisation" % (w.n_layers, w.n_layers, w.n_layers),
            "eager_value": replica_throughput(B * e2e_steps, timings["eager"], world, device)[0],
-           "eager_path": "the same with the 32 pp_layer calls made eagerly every step"}
+           "eager_path": "the same with the %d pp_layer calls made eagerly every step" % w.n_layers}
 
     # ---- router statistics (L_ent, L_bal, L_gate) over a batch of 8192 tokens' logits
     T_st = 8192
@@ -575,59 +641,78 @@ def main():
     us_st = e0.elapsed_time(e1) * 1e3 / n_st
     router_stats = {"tokens": T_st, "experts": w.n_experts, "us_per_call": us_st,
                     "gbs": T_st * w.n_experts * 4 / (us_st * 1e-6) / 1e9,
-                    "note": "two launches (per-256-token parts, fixed-order final sum); logits L2-resident"}
+                    "note": "two launches (per-block parts, fixed-order final sum); logits L2-resident"}
 
     # ---- MoEfication repacking (Eq. permuted_weights) of one layer's weights by a random permutation
-    moefy_permute = None
-    if not args.skip_extras:
-        L0 = layers[0]
-        perm_d = torch.randperm(w.d_ff, device=device).to(torch.int32)
-        outs = [None if L0["Wg"] is None else torch.empty_like(L0["Wg"]), torch.empty_like(L0["Wu"]),
-                torch.empty_like(L0["Wd"])]
-        ws_mp = pp.alloc_workspace(desc, 0)
-        with torch.cuda.stream(stream):
-            for _ in range(3):
-                pp.pp_moefy_permute(desc, perm_d, L0["Wg"], L0["Wu"], L0["Wd"], *outs, ws_mp, stream=stream)
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            n_mp = 20
-            e0.record(stream)
-            for _ in range(n_mp):
-                pp.pp_moefy_permute(desc, perm_d, L0["Wg"], L0["Wu"], L0["Wd"], *outs, ws_mp, stream=stream)
-            e1.record(stream)
-            stream.synchronize()
-        if pp.pp_get_device_status(ws_mp) != pp.PP_OK:
-            raise SystemExit("device status after the repacking leg: %s" % pp.status_name(pp.pp_get_device_status(ws_mp)))
-        pl = perm_d.long()
-        ok = torch.equal(outs[1][:64], L0["Wu"][pl[:64]]) and torch.equal(outs[2][:, :64], L0["Wd"][:, pl[:64]])
-        us_mp = e0.elapsed_time(e1) * 1e3 / n_mp
-        n_mat = 3 if L0["Wg"] is not None else 2
-        b_mp = 2 * n_mat * w.d_ff * w.d_model * L0["Wu"].element_size()
-        moefy_permute = {"us_per_call": us_mp, "bytes": b_mp, "gbs": b_mp / (us_mp * 1e-6) / 1e9,
-                         "frac_of_hbm_peak": b_mp / (us_mp * 1e-6) / 1e9 / hbm_peak, "spot_check": bool(ok),
-                         "what": "pp_moefy_permute of one layer (W_gate/W_up rows, W_down columns) by a random "
-                                 "permutation; bytes = read + write of the three matrices; 3 launches per call"}
-        del outs, ws_mp
+    L0 = layers[0]
+    perm_d = torch.randperm(w.d_ff, device=device).to(torch.int32)
+    outs = [None if L0["Wg"] is None else torch.empty_like(L0["Wg"]), torch.empty_like(L0["Wu"]),
+            torch.empty_like(L0["Wd"])]
+    ws_mp = pp.alloc_workspace(desc, 0)
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            pp.pp_moefy_permute(desc, perm_d, L0["Wg"], L0["Wu"], L0["Wd"], *outs, ws_mp, stream=stream)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        n_mp = 20
+        e0.record(stream)
+        for _ in range(n_mp):
+            pp.pp_moefy_permute(desc, perm_d, L0["Wg"], L0["Wu"], L0["Wd"], *outs, ws_mp, stream=stream)
+        e1.record(stream)
+        stream.synchronize()
+    if pp.pp_get_device_status(ws_mp) != pp.PP_OK:
+        raise SystemExit("device status after the repacking leg: %s" % pp.status_name(pp.pp_get_device_status(ws_mp)))
+    pl = perm_d.long()
+    ok = torch.equal(outs[1][:64], L0["Wu"][pl[:64]]) and torch.equal(outs[2][:, :64], L0["Wd"][:, pl[:64]])
+    us_mp = e0.elapsed_time(e1) * 1e3 / n_mp
+    n_mat = 3 if L0["Wg"] is not None else 2
+    b_mp = 2 * n_mat * w.d_ff * w.d_model * L0["Wu"].element_size()
+    moefy_permute = {"us_per_call": us_mp, "bytes": b_mp, "gbs": b_mp / (us_mp * 1e-6) / 1e9,
+                     "frac_of_hbm_peak": b_mp / (us_mp * 1e-6) / 1e9 / load_peaks()[0], "spot_check": bool(ok),
+                     "what": "pp_moefy_permute of one layer (W_gate/W_up rows, W_down columns) by a random "
+                             "permutation; bytes = read + write of the three matrices"}
+    del outs, ws_mp, head, layers, desc, ws
+    torch.cuda.empty_cache()
+
+    # ---- the other workload shapes: each timed on its own, with its own roofline and clocks
+    configs = {}
+    for item in [v for v in args.configs.split(",") if v]:
+        parts = item.split(":")
+        cw = wl.WORKLOADS[parts[0]]
+        cB, cp = int(parts[1]), float(parts[2])
+        if len(parts) > 3:
+            from dataclasses import replace
+            cw = replace(cw, n_layers=int(parts[3]))
+        full_layers = wl.WORKLOADS[parts[0]].n_layers
+        cpool = default_pool(cB)
+        m = measure(pp, cw, cB, cp, args.config_steps, max(args.warmup, 5), cpool, args.seed, device, stream,
+                    flush, world)
+        rec = public(m)
+        rec["config"] = config_dict(cw, cB, cp, cpool, world, args.no_flush)
+        rec["gpu_launches"] = m["launches"] * (1 if path_kind(cw, cB) == "decode" else 9)
+        if cw.n_layers != full_layers:
+            rec["model_tokens_per_s"] = m["tokens_per_s"] * cw.n_layers / full_layers
+            rec["scaling_note"] = ("timed on %d of the model's %d layers (same shape, independently drawn); "
+                                   "model_tokens_per_s = tokens_per_s x %d / %d, layers running back to back"
+                                   % (cw.n_layers, full_layers, cw.n_layers, full_layers))
+        configs["%s@B%d@p%g" % (cw.name, cB, cp)] = rec
+        del m
+        torch.cuda.empty_cache()
 
     out = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-           "config": {"workload": w.name, "d_model": w.d_model, "d_ff": w.d_ff, "n_experts": w.n_experts,
-                      "d_expert": 64, "layers": w.n_layers, "batch": B, "p": args.p, "act": w.act,
-                      "token_pool": args.pool,
-                      "l2": "no flush (warm)" if args.no_flush else "flushed between steps (256 MiB write, untimed)",
-                      "parallelism": "replicas" if world > 1 else "single GPU"},
-           "roofline": dict(roof, achieved=achieved, peak=peak, frac=achieved / peak,
-                            traffic=kernel_traffic(w.name, args.p, B, "decode" if B <= 4 or w.dtype == "f32" else "grouped"),
-                            peak_kind=peak_kind,
-                            kernel="decode_layer_kernel" if B <= 4 else "pp_layer (grouped tcgen05 path)",
-                            per="one pp_layer call (one layer)", launch_ms=per_launch_ms),
-           "expert_bytes": {"gbs": expert_gbs, "frac_of_peak": expert_gbs / hbm_peak,
-                            "frac_of_8tbs": expert_gbs / 8000.0, "k_mean": k_mean, "k_min": int(ks.min()),
-                            "k_max": int(ks.max()), "s_ffn": s_ffn},
-           "hbm_gbs_total": tot_b / seconds / 1e9, "tflops": tot_f / seconds / 1e12,
+           "config": config_dict(w, B, args.p, args.pool, world, args.no_flush),
+           "roofline": roof,
+           "expert_bytes": {"gbs": head_rec["expert_gbs"], "frac_of_peak": head_rec["expert_gbs"] / load_peaks()[0],
+                            "frac_of_8tbs": head_rec["expert_gbs"] / 8000.0, "k_mean": head_rec["k_mean"],
+                            "k_min": head_rec["k_min"], "k_max": head_rec["k_max"],
+                            "union_mean": head_rec["union_mean"], "s_ffn": head_rec["s_ffn"],
+                            "s_ffn_from": head_rec["s_ffn_from"]},
+           "hbm_gbs_total": head_rec["total_gbs"], "tflops": head_rec["tflops"],
            "p_sweep": sweep, "rules": rules, "chained": chained, "router_stats": router_stats,
            "moefy_permute": moefy_permute, "warm_l2_tokens_per_s": warm_tok_s,
-           "e2e": e2e, "gpu_launches": launches * kernels_per_layer, "clocks": clocks}
+           "e2e": e2e, "gpu_launches": args.steps * w.n_layers * kernels_per_layer, "clocks": head_rec["clocks"],
+           "configs": configs}
     if rank == 0 and world == 1:
         try:
             out["cpu_baseline"] = run_oracle_sample(w, args.cpu_seconds, args.seed, p=args.p, B=B)

@@ -182,7 +182,8 @@ pp_status pp_layer_chained(const pp_desc *desc, const void *x_prev, const void *
    that exposes no allocator.  The paper has no counterpart: this entry point
    exists only for those callers.
    Same computation and arguments as pp_layer, for T <= 4 tokens and without a
-   workspace.  Its scratch (status word, per-CTA launch counts, router
+   workspace.  Like pp_layer, it runs the tokens in slices when one fused
+   launch cannot hold them all (fp32 rows of a wide model).  Its scratch (status word, per-CTA launch counts, router
    logits and gate/up activations: 533,760 bytes) is one static
    device array that every GPU loading this library keeps until the process
    exits; no call allocates or frees.

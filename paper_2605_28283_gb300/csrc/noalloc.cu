@@ -129,35 +129,32 @@ extern "C" pp_status pp_layer_noalloc(const pp_desc* desc, const void* x, int T,
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     const pp_desc& d = *desc;
 
+    // The largest token count one fused launch takes for this shape (pp_layer
+    // does the same): fp32 rows of a wide model may fit shared memory only
+    // one token at a time.  T is then run in slices of that many tokens.
     int TS = 1;
     while (TS < T) TS <<= 1;
     pp::DecodePlan plan;
-    const pp::DecodePlanIn in{d.dtype, d.d_model, d.n_experts, TS, ds->sms, d.act == PP_ACT_SWIGLU,
-                              ds->smem_optin - pp::kDecodeStaticSmemReserve};
-    if (!pp::decode_plan(in, &plan)) return PP_ERR_SHAPE;
+    for (;; TS >>= 1) {
+        if (TS < 1) return PP_ERR_SHAPE;
+        const pp::DecodePlanIn in{d.dtype, d.d_model, d.n_experts, TS, ds->sms, d.act == PP_ACT_SWIGLU,
+                                  ds->smem_optin - pp::kDecodeStaticSmemReserve};
+        if (pp::decode_plan(in, &plan)) break;
+    }
 
     pp::DecodeArgs a;
     std::memset(&a, 0, sizeof a);
     if (!encode_down_map(d, W_down, plan.R6, &a.tmap_down)) return PP_ERR_CUDA;
     unsigned char* scratch = ds->scratch;
     pp::Control* ctl = reinterpret_cast<pp::Control*>(scratch);
-    a.x = x;
     a.Wr = W_r;
     a.Wg = W_gate;
     a.Wu = W_up;
-    a.y = y;
-    if (sel_out) {
-        a.sel_ids = sel_out->ids;
-        a.sel_counts = sel_out->counts;
-        a.sel_gates = sel_out->gates;
-        a.sel_logits = sel_out->logits;
-    }
     a.tlog = reinterpret_cast<unsigned long long*>(scratch + kCtlBytes);
     a.th = reinterpret_cast<unsigned long long*>(scratch + kCtlBytes + kLogitBytes);
     a.epochs = ctl->epoch;
     a.status = &ctl->status;
     a.timeout_ns = kTimeoutNs;
-    a.T = T;
     a.d = d.d_model;
     a.E = d.n_experts;
     a.act = d.act;
@@ -181,9 +178,23 @@ extern "C" pp_status pp_layer_noalloc(const pp_desc* desc, const void* x, int T,
     a.off_ring4 = plan.off_ring4;
 
     // The status word starts at zero for every call.  The launch counts and the tagged words carry over from call to
-    // call (zero at load time): a call only accepts words tagged by itself.
+    // call (zero at load time): a launch only accepts words tagged by itself.
     if (cudaMemsetAsync(&ctl->status, 0, sizeof(unsigned), st) != cudaSuccess) return PP_ERR_CUDA;
-    if (pp::decode_launch(a, plan, d.dtype, TS, ds->sms, st) != cudaSuccess) return PP_ERR_CUDA;
+    const size_t esz = d.dtype == PP_BF16 ? 2 : 4;
+    const size_t E = (size_t)d.n_experts;
+    for (int t0 = 0; t0 < T; t0 += TS) {
+        const int n = T - t0 < TS ? T - t0 : TS;  // the kernel instance for TS tokens takes any n <= TS
+        a.T = n;
+        a.x = static_cast<const char*>(x) + (size_t)t0 * d.d_model * esz;
+        a.y = static_cast<char*>(y) + (size_t)t0 * d.d_model * esz;
+        if (sel_out) {
+            a.sel_ids = sel_out->ids + (size_t)t0 * E;
+            a.sel_counts = sel_out->counts + t0;
+            a.sel_gates = sel_out->gates + (size_t)t0 * E;
+            a.sel_logits = sel_out->logits ? sel_out->logits + (size_t)t0 * E : nullptr;
+        }
+        if (pp::decode_launch(a, plan, d.dtype, TS, ds->sms, st) != cudaSuccess) return PP_ERR_CUDA;
+    }
     if (status_out &&
         cudaMemcpyAsync(status_out, &ctl->status, sizeof(uint32_t), cudaMemcpyDeviceToDevice, st) != cudaSuccess)
         return PP_ERR_CUDA;

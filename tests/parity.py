@@ -1,7 +1,8 @@
 """Helpers for the GPU-vs-oracle parity tests.
 
 Inputs come from the seeded host recipe in ``paper_2605_28283_gb300.workloads``;
-expected values come only from the CPU oracle.  Bars (spec contract):
+expected values come only from the CPU oracle, and every GPU value is taken
+through the library's C ABI.  The bars:
 
 * selection, identical logits (pp_select): counts and ids bit-exact, except
   "boundary" tokens whose oracle prefix mass S_i (LTE: a sigmoid score) lies

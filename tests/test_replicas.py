@@ -33,12 +33,19 @@ def _rank_main(rank, world, port, results):
 
     class Args:
         workload, batch, seed, p, steps, warmup, gpus = "tiny_relu_f32", 2, 0, 0.7, 2, 1, world
+        pool, no_flush = 64, False
 
     out = io.StringIO()
     with redirect_stdout(out):
         bench.run_reference(Args())
     results[rank] = (r, w, value, slowest, out.getvalue())
     dist.destroy_process_group()
+
+
+def bench_workload(name):
+    sys.path.insert(0, ROOT)
+    from paper_2605_28283_gb300 import workloads as wl
+    return wl.WORKLOADS[name]
 
 
 def test_two_replicas_report_all_tokens_over_the_slowest_rank():
@@ -57,4 +64,8 @@ def test_two_replicas_report_all_tokens_over_the_slowest_rank():
     assert len(lines) == 1
     rec = json.loads(lines[0])
     assert rec["impl"] == "reference" and rec["cpu_baseline"]["kind"] == "oracle" and rec["value"] > 0
+    # the reference arm states its host cores and prints the GPU arm's config dict
+    assert {"cpu_count", "affinity_cores", "omp_threads"} <= set(rec["cpu_baseline"])
+    import bench
+    assert rec["config"] == bench.config_dict(bench_workload("tiny_relu_f32"), 2, 0.7, 64, 2, False)
     assert res[1][4].strip() == ""

@@ -49,6 +49,29 @@ def test_noalloc_matches_pp_layer(pp, name, T, p):
         assert err.max() <= Y_TOL[w.dtype], (call, float(err.max()))
 
 
+def test_noalloc_slices_wide_fp32_rows(pp):
+    """fp32 rows of d_model = 8192 fit the fused kernel's shared memory one
+    token at a time: both entry points run such a call in one-token slices."""
+    import torch
+    w, L = layer_inputs("tiny_relu_f32", 3, d=8192, E=16)
+    desc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act)
+    x, Wr, Wu, Wd = dev(L.x), dev(L.Wr), dev(L.Wu), dev(L.Wd)
+    ws = pp.alloc_workspace(desc, 3)
+    ref_sel = pp.Selection.empty(3, w.n_experts, "cuda")
+    y_ref = torch.empty_like(x)
+    pp.pp_layer(desc, x, 3, Wr, None, Wu, Wd, f32(0.7), ref_sel, y_ref, ws)
+    for call in range(2):
+        sel = pp.Selection.empty(3, w.n_experts, "cuda")
+        y = torch.full_like(x, float("nan"))
+        status = torch.full((1,), -1, dtype=torch.int32, device="cuda")
+        pp.pp_layer_noalloc(desc, x, 3, Wr, None, Wu, Wd, f32(0.7), sel, y, status)
+        torch.cuda.synchronize()
+        assert int(status.item()) == pp.PP_OK
+        np.testing.assert_array_equal(to_host(sel.counts), to_host(ref_sel.counts))
+        np.testing.assert_array_equal(to_host(sel.ids), to_host(ref_sel.ids))
+        assert rel_err_per_token(to_host(y), to_host(y_ref)).max() <= Y_TOL["f32"]
+
+
 def test_noalloc_without_selection_output(pp):
     import torch
     w, L = layer_inputs("llama2_7b_decode", 1)
