@@ -319,6 +319,9 @@ def measure(pp, w, B, p, steps, warmup, pool, seed, device, stream, flush, world
     ws = pp.alloc_workspace(desc, B)
     if layers is None:
         layers = make_layers(w, B, pool, seed, device)
+    # the workspace is zeroed and the inputs drawn on torch's current stream;
+    # the library's launches go to `stream`
+    torch.cuda.synchronize()
     pf = float(np.float32(p))
     graphs = capture_graphs(pp, desc, layers, pf, B, pool, ws, stream)
     sampler = ClockSampler(torch.cuda.current_device()) if clocks else None
@@ -628,6 +631,7 @@ def main():
     g_st = torch.randn((T_st, w.n_experts), device=device) * 3.0
     ws_st = pp.alloc_workspace(desc, T_st)
     out_st = torch.empty(3, dtype=torch.float64, device=device)
+    torch.cuda.synchronize()  # inputs and workspace were made on torch's current stream
     with torch.cuda.stream(stream):
         for _ in range(5):
             pp.pp_router_stats(desc, g_st, T_st, 1e-9, out_st, ws_st, stream=stream)
@@ -649,6 +653,7 @@ def main():
     outs = [None if L0["Wg"] is None else torch.empty_like(L0["Wg"]), torch.empty_like(L0["Wu"]),
             torch.empty_like(L0["Wd"])]
     ws_mp = pp.alloc_workspace(desc, 0)
+    torch.cuda.synchronize()
     with torch.cuda.stream(stream):
         for _ in range(3):
             pp.pp_moefy_permute(desc, perm_d, L0["Wg"], L0["Wu"], L0["Wd"], *outs, ws_mp, stream=stream)
