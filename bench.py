@@ -55,6 +55,8 @@ def parse():
     ap.add_argument("--configs", default="llama3_8b_batched:64:0.7,llama2_13b_prefill:8192:0.7:1,gpt2m_gelu_bf16:4:0.7",
                     help="further workloads timed after the headline, workload:batch:p[:layers] ('' = none)")
     ap.add_argument("--config-steps", type=int, default=300)
+    ap.add_argument("--timeline", action="store_true",
+                    help="phase timeline of the fused decode kernel (B = 1) instead of the benchmark")
     return ap.parse_args()
 
 
@@ -460,6 +462,105 @@ def run_reference(args):
     print(json.dumps(out))
 
 
+# -------------------------------------------------------------- timeline
+STAMP_NAMES = ["entry", "released", "x", "router", "selected", "union", "issued4", "phase4", "first_h", "phase6",
+               "end", "logits_in", "cut", "cand", "landed4"]
+
+
+def timeline_summary(st):
+    """st: [steps, layers, CTAs, 16] global-timer stamps (0 = phase skipped).
+    Per launch, times are taken from the first CTA's release (the previous
+    grid on the stream complete).  The timer advances in steps of a few
+    hundred ns, so per phase the mean over CTAs (and the mean of the
+    per-launch maximum) is reported, averaged over launches, in
+    microseconds; also the gap from one launch's last CTA end to the next
+    launch's release."""
+    import numpy as np
+    rows = {n: ([], []) for n in STAMP_NAMES}
+    gaps = []
+    S, L = st.shape[0], st.shape[1]
+    for s in range(S):
+        prev_end = None
+        for l in range(L):
+            a = st[s, l].astype(np.float64)
+            rel = a[:, 1][a[:, 1] > 0]
+            if rel.size == 0:
+                continue
+            t0 = rel.min()
+            for i, n in enumerate(STAMP_NAMES):
+                v = a[:, i][a[:, i] > 0]
+                if v.size:
+                    rows[n][0].append(np.mean(v - t0) / 1e3)
+                    rows[n][1].append((v - t0).max() / 1e3)
+            if prev_end is not None:
+                gaps.append((t0 - prev_end) / 1e3)
+            ends = a[:, 10][a[:, 10] > 0]
+            prev_end = ends.max() if ends.size else None
+    out = {n: {"mean_cta_us": float(np.mean(m)), "last_cta_us": float(np.mean(x))}
+           for n, (m, x) in rows.items() if m}
+    out["gap_last_end_to_next_release_us"] = float(np.mean(gaps)) if gaps else None
+    return out
+
+
+def run_timeline(args):
+    """Headline workload (B = 1) through pp_debug_decode_timeline: the same
+    kernel as pp_layer plus global-timer stamps at its phase boundaries; L
+    layers per step back to back in one CUDA graph, as in the benchmark."""
+    import numpy as np
+    import torch
+    from paper_2605_28283_gb300 import binding as pp
+    from paper_2605_28283_gb300 import workloads as wl
+    torch.cuda.set_device(0)
+    device = torch.device("cuda", 0)
+    pp.load()
+    w = wl.WORKLOADS[args.workload]
+    if args.layers:
+        from dataclasses import replace
+        w = replace(w, n_layers=args.layers)
+    pool = min(args.pool, 16)
+    layers = make_layers(w, 1, pool, args.seed, device)
+    desc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act)
+    ws = pp.alloc_workspace(desc, 1)
+    stamps = torch.zeros((w.n_layers, 256 * 16), dtype=torch.int64, device=device)
+    flush = None if args.no_flush else torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=device)
+    stream = torch.cuda.Stream()
+    pf = float(np.float32(args.p))
+    torch.cuda.synchronize()
+
+    def step(i):
+        for l, L in enumerate(layers):
+            pp.pp_debug_decode_timeline(desc, L["x"][i], L["Wr"], L["Wg"], L["Wu"], L["Wd"], pf, L["y"], ws,
+                                        stamps[l], stream=stream)
+    graphs = []
+    with torch.cuda.stream(stream):
+        for i in range(pool):
+            step(i)
+        stream.synchronize()
+        for i in range(pool):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                step(i)
+            graphs.append(g)
+        for i in range(args.warmup):
+            graphs[i % pool].replay()
+        out = []
+        for i in range(args.steps):
+            stamps.zero_()
+            if flush is not None:
+                flush.add_(1)
+            graphs[i % pool].replay()
+            stream.synchronize()
+            out.append(stamps.view(w.n_layers, 256, 16).cpu().numpy())
+    if pp.pp_get_device_status(ws) != pp.PP_OK:
+        raise SystemExit("device status: %s" % pp.status_name(pp.pp_get_device_status(ws)))
+    sm = torch.cuda.get_device_properties(0).multi_processor_count
+    st = np.stack(out)[:, :, :sm, :]
+    res = {"what": "decode_layer_kernel phase timeline (timeline instantiation, one stamp set per CTA)",
+           "workload": w.name, "layers": w.n_layers, "p": args.p, "steps": args.steps, "token_pool": pool,
+           "l2": "no flush" if args.no_flush else "flushed between steps", "phases": timeline_summary(st)}
+    print(json.dumps(res))
+
+
 # ------------------------------------------------------------------ main
 def public(m):
     """A measurement record without its device objects."""
@@ -472,6 +573,8 @@ def main():
         args.pool = default_pool(args.batch)
     if args.impl == "reference":
         return run_reference(args)
+    if args.timeline:
+        return run_timeline(args)
     import numpy as np
     import torch
     rank, world, local = dist_env()

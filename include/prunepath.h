@@ -271,6 +271,21 @@ pp_status pp_moefy_permute(const pp_desc *desc, const int32_t *perm, const void 
 /* Synchronise `stream` and return the sticky device status of `ws`. */
 pp_status pp_get_device_status(void *ws, void *stream);
 
+/* Diagnostic: pp_layer for one bf16 token (T = 1) through the timeline
+   instantiation of the fused decode kernel, which computes the same y and
+   also records the GPU global timer (ns) at the phase boundaries of every
+   CTA: stamps[CTA * 16 + i] for i = first instruction, preceding grid
+   complete, x loaded, router logits published, selection made, union formed,
+   gate/up loads issued, gate/up activations published, first activations of
+   the down projection received, down products done, y written (0 where a CTA
+   skips a phase: the caller zeroes stamps first, so that consecutive layers
+   need nothing between their launches).  stamps: device uint64, at least
+   256 * 16 entries (stamps_bytes).  Errors as pp_layer; a dtype
+   other than bf16 is PP_ERR_DTYPE. */
+pp_status pp_debug_decode_timeline(const pp_desc *desc, const void *x, const void *W_r, const void *W_gate,
+                                   const void *W_up, const void *W_down, float p, void *y, void *ws,
+                                   size_t ws_bytes, uint64_t *stamps, size_t stamps_bytes, void *stream);
+
 /* Test hook for failure detection: enqueue one kernel that waits on a
    workspace flag nothing sets, with a limit of timeout_ns nanoseconds; it
    then records PP_ERR_TIMEOUT in the workspace status and returns.  No GPU

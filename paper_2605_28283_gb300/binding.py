@@ -63,6 +63,7 @@ EXPORTS = {
     "pp_moefy_permute": (_I, [_PD, _P, _P, _P, _P, _P, _P, _P, _P, _Z, _P]),
     "pp_get_device_status": (_I, [_P, _P]),
     "pp_debug_wait_timeout": (_I, [_P, _Z, _LL, _P]),
+    "pp_debug_decode_timeline": (_I, [_PD, _P, _P, _P, _P, _P, _F, _P, _P, _Z, _P, _Z, _P]),
     "pp_status_string": (ctypes.c_char_p, [_I]),
     "pp_version": (ctypes.c_char_p, []),
 }
@@ -249,6 +250,14 @@ def pp_moefy_permute(desc, perm, W_gate, W_up, W_down, W_gate_out, W_up_out, W_d
 
 def pp_get_device_status(ws, stream=None) -> int:
     return int(load().pp_get_device_status(_ptr(ws), _stream(stream)))
+
+
+def pp_debug_decode_timeline(desc, x, W_r, W_gate, W_up, W_down, p, y, ws, stamps, stream=None):
+    """stamps: a device uint64 tensor of at least 256 * 16 entries."""
+    _check(load().pp_debug_decode_timeline(ctypes.byref(desc), _ptr(x), _ptr(W_r), _ptr(W_gate), _ptr(W_up),
+                                           _ptr(W_down), float(p), _ptr(y), *_wsargs(ws), _ptr(stamps),
+                                           stamps.numel() * stamps.element_size(), _stream(stream)),
+           "pp_debug_decode_timeline")
 
 
 def pp_debug_wait_timeout(ws, timeout_ns, stream=None):

@@ -265,7 +265,8 @@ GroupedArgs grouped_args(const pp_desc& d, int T, void* ws, const void* x, const
 // One launch of the fused decode kernel over tokens [t0, t0 + n).
 pp_status decode_call(const pp_desc& d, const void* x, int t0, int n, const void* Wr, const void* Wg,
                       const void* Wu, const void* Wd, float p, const pp_selection* sel, bool do_route,
-                      bool do_ffn, void* y, const Ws& w, cudaStream_t st, const Chain* chain = nullptr) {
+                      bool do_ffn, void* y, const Ws& w, cudaStream_t st, const Chain* chain = nullptr,
+                      unsigned long long* tline = nullptr) {
     const DeviceInfo di = device_info();
     int TS = 1;
     while (TS < n) TS <<= 1;
@@ -324,6 +325,7 @@ pp_status decode_call(const pp_desc& d, const void* x, int t0, int n, const void
         a.x_out = static_cast<char*>(chain->x_out) + (size_t)t0 * d.d_model * esz;
         a.eps = chain->eps;
     }
+    a.tline = tline;
     return cuda_status(decode_launch(a, plan, d.dtype, TS, di.sms, st));
 }
 
@@ -612,6 +614,26 @@ pp_status pp_get_device_status(void* ws, void* stream) {
         return PP_ERR_CUDA;
     if (cudaStreamSynchronize(st) != cudaSuccess) return PP_ERR_CUDA;
     return static_cast<pp_status>(v);
+}
+
+pp_status pp_debug_decode_timeline(const pp_desc* desc, const void* x, const void* W_r, const void* W_gate,
+                                    const void* W_up, const void* W_down, float p, void* y, void* ws, size_t ws_bytes,
+                                    uint64_t* stamps, size_t stamps_bytes, void* stream) {
+    PP_TRY(check_desc(desc));
+    if (desc->dtype != PP_BF16) return PP_ERR_DTYPE;
+    if (std::isnan(p)) return PP_ERR_INVALID_ARG;
+    if (!x || !y || !W_r || !stamps) return PP_ERR_INVALID_ARG;
+    if (!aligned16(x) || !aligned16(y) || !aligned16(W_r) || !aligned16(stamps)) return PP_ERR_ALIGN;
+    PP_TRY(check_weights(desc, W_gate, W_up, W_down));
+    PP_TRY(check_ws(desc, 1, ws, ws_bytes));
+    PP_TRY(check_device());
+    if (stamps_bytes < (size_t)kMaxGrid * kDecodeStamps * sizeof(uint64_t)) return PP_ERR_INVALID_ARG;
+    if (decode_ts_limit(*desc) < 1) return PP_ERR_SHAPE;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const Ws w = ws_views(*desc, 1, ws);
+    const float kp = rule_kernel_param(desc->rule, p, desc->n_experts);
+    return decode_call(*desc, x, 0, 1, W_r, W_gate, W_up, W_down, kp, nullptr, true, true, y, w, st, nullptr,
+                       reinterpret_cast<unsigned long long*>(stamps));
 }
 
 pp_status pp_debug_wait_timeout(void* ws, size_t ws_bytes, long long timeout_ns, void* stream) {

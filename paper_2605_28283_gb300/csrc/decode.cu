@@ -43,8 +43,10 @@ constexpr int kBarX = 0, kBarR = 1, kBarFull4 = 2, kBarFull6 = kBarFull4 + kMaxN
               kBarH = kBarFull6 + kWarps * kMaxSlots6, kNumBars = kBarH + kWarps;
 
 // Selection given by the caller (pp_sparse_ffn): gates are summed per expert
-// so repeated ids behave like repeated terms of the sum.
-PP_DEVINL void load_given_selection(const DecodeArgs& a, float* gw, unsigned* mask) {
+// so repeated ids behave like repeated terms of the sum.  (Like the other
+// paths that the fused layer does not take, kept out of line: the kernel
+// runs once per launch and is bound by instruction fetch.)
+static __device__ __noinline__ void load_given_selection(const DecodeArgs& a, float* gw, unsigned* mask) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (warp >= a.T) return;
     const int t = warp, E = a.E;
@@ -64,9 +66,46 @@ PP_DEVINL void load_given_selection(const DecodeArgs& a, float* gw, unsigned* ma
     }
 }
 
+// Selection of every token by the whole CTA, in turn, from the tagged logits
+// as they arrive, for the rules other than the cumulative-mass cut (top-k,
+// LTE's threshold, p >= 1); CTA 0 publishes it.  Out of line, like
+// load_given_selection.
+static __device__ __noinline__ void decode_select_cta(const DecodeArgs& a, unsigned tag, float* gw, unsigned* mask,
+                                                      CtaSelScratch& sc) {
+    const int tid = threadIdx.x, T = a.T, E = a.E;
+    const bool publish = blockIdx.x == 0;
+    const bool want_rank = publish && a.sel_ids != nullptr;
+    for (int t = 0; t < T; t++) {
+        bool on;
+        int r;
+        float g;
+        const unsigned long long* row = a.tlog + (size_t)t * E;
+        const int k = cta_select_fn([&](int j) { return wait_tagged(row + j, tag, a.status, a.timeout_ns); }, E, a.p,
+                                    a.rule, want_rank, sc, a.status, &on, &r, &g);
+        const int j = tid;
+        if (j < E) {
+            const float gv = on ? (a.gate == PP_GATE_NONE ? 1.0f : sigmoidf_(g)) : 0.0f;
+            if (on) {
+                gw[t * E + j] = gv;
+                mask[j] |= 1u << t;
+            }
+            if (publish) {
+                if (a.sel_ids)
+                    write_selection_row(a.sel_ids + (size_t)t * E, a.sel_gates + (size_t)t * E, j, E, k, on, r, gv);
+                if (a.sel_logits) a.sel_logits[(size_t)t * E + j] = g;
+            }
+        }
+        if (publish && tid == 0 && a.sel_counts) a.sel_counts[t] = k;
+        __syncthreads();  // scratch reuse by the next token
+    }
+}
+
 // CHAIN: the chained step's prologue (a.chain) is compiled only into its own
 // instantiations, so that the plain layer's kernel carries no extra code.
-template <typename TW, int TS, int RPL, bool CHAIN>
+// TL: the timeline instantiation, which also records the global timer at
+// the phase boundaries of every CTA into a.tline[CTA][kDecodeStamps] (a
+// diagnostic; the plain kernel has no such stores).
+template <typename TW, int TS, int RPL, bool CHAIN, bool TL>
 __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __grid_constant__ DecodeArgs a) {
     extern __shared__ __align__(1024) unsigned char smem[];
     using EL = Elem<TW>;
@@ -89,9 +128,26 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     unsigned char* ring4 = smem + a.off_ring4;
     unsigned char* ring6 = smem + a.off_ring6;
     __shared__ __align__(16) CtaSelScratch sel_sc;
+    __shared__ __align__(16) CutShared cut_sc;
     __shared__ int s_nU;
     __shared__ int s_wcount[kWarps];
     __shared__ unsigned s_tag;
+    __shared__ int s_k[TS];  // activated experts per token (cumulative-mass cut)
+    // timeline stamp i of this CTA (TL instantiation, called by thread 0 only):
+    // the global timer at entry, then that plus the SM cycles since entry at
+    // kStampMHz (the global timer advances in steps of a few hundred ns)
+    uint64_t g0 = 0;
+    long long c0 = 0;
+    auto stamp = [&](int i) {
+        if constexpr (TL)
+            a.tline[(size_t)b * kDecodeStamps + i] =
+                g0 + (unsigned long long)((clock64() - c0) * 1000ll / kStampMHz);
+    };
+    if (TL && tid == 0) {
+        c0 = clock64();
+        g0 = globaltimer_ns();
+        stamp(kStEntry);
+    }
 
     if (tid == 0) {
         for (int i = 0; i < kNumBars; i++) mbar_init(&bars[i], 1);
@@ -99,6 +155,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     }
     for (int i = tid; i < TS * E; i += kDecThreads) gw[i] = 0.0f;
     for (int i = tid; i < kMaxExperts; i += kDecThreads) mask[i] = 0u;
+    if (tid < TS) s_k[tid] = 0;
     __syncthreads();
 
     // this CTA's router rows [j0, j1) of W_r (phase 1)
@@ -118,6 +175,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     }
     pdl_wait();
     pdl_launch_dependents();
+    if (TL && tid == 0) stamp(kStReleased);
     TW* chain_y = reinterpret_cast<TW*>(ring4 + a.off_chain);
     TW* chain_g = chain_y + (size_t)TS * d;
     if (tid == 0) {
@@ -138,6 +196,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     mbar_wait(&bars[kBarX], 0, a.status, lim);
     __syncthreads();
     const unsigned tag = s_tag;
+    if (TL && tid == 0) stamp(kStX);
 
     // chained step: the layer input is RMSNorm(x_prev + y_prev) * gamma, formed
     // in place in shared memory by every CTA (CTA 0 also stores it)
@@ -180,6 +239,25 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
             __syncthreads();  // red is reused by the next token
         }
     }
+
+    // gate/up rows of global neuron q (neuron q & 63 of the expert at
+    // position q >> 6 of U) -> phase-4 ring slot `slot`
+    const uint32_t stage4 = (uint32_t)((gated ? 2 : 1) * rowb);
+    const TW* Wg = reinterpret_cast<const TW*>(a.Wg);
+    const TW* Wu = reinterpret_cast<const TW*>(a.Wu);
+    auto issue_row = [&](int q, int slot) {
+        const size_t row = (size_t)ulist[q >> 6] * kDExpert + (q & 63);
+        unsigned char* dst = ring4 + (size_t)slot * stage4;
+        uint64_t* fb = &bars[kBarFull4 + slot];
+        mbar_arrive_expect_tx(fb, stage4);
+        if (gated) {
+            bulk_g2s(dst, Wg + row * d, (uint32_t)rowb, fb);
+            bulk_g2s(dst + rowb, Wu + row * d, (uint32_t)rowb, fb);
+        } else {
+            bulk_g2s(dst, Wu + row * d, (uint32_t)rowb, fb);
+        }
+    };
+    const bool mass_cut = (a.rule == PP_SEL_MIN_PREFIX || a.rule == PP_SEL_PAPER) && a.p < 1.0f;
 
     // ---------------------------------------------------------- phase 1
     if (a.do_route) {
@@ -228,42 +306,79 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
                 __syncthreads();
             }
         }
-        // selection of every token by the whole CTA, from the tagged logits
-        // as they arrive; CTA 0 publishes it
+        if (TL && tid == 0) stamp(kStRouter);
         const bool publish = b == 0;
-        const bool want_rank = publish && a.sel_ids != nullptr;
-        for (int t = 0; t < T; t++) {
-            bool on;
-            int r;
-            float g;
-            const unsigned long long* row = a.tlog + (size_t)t * E;
-            const int k = cta_select_fn([&](int j) { return wait_tagged(row + j, tag, a.status, lim); }, E, a.p,
-                                        a.rule, want_rank, sel_sc, a.status, &on, &r, &g);
-            const int j = tid;
-            if (j < E) {
-                const float gv = on ? (a.gate == PP_GATE_NONE ? 1.0f : sigmoidf_(g)) : 0.0f;
-                if (on) {
-                    gw[t * E + j] = gv;
-                    mask[j] |= 1u << t;
+        if (mass_cut) {
+            // cumulative-mass cut of every token by the whole CTA (thread j
+            // waits for logit j); every activated expert is recorded by the
+            // thread that decides it
+            // candidate scratch in the phase-6 ring, idle until phase 6: the
+            // phase-4 ring takes gate/up rows requested during the count
+            WarpCand* cand = reinterpret_cast<WarpCand*>(ring6);
+            for (int t = 0; t < T; t++) {
+                const float g = tid < E ? wait_tagged(a.tlog + (size_t)t * E + tid, tag, a.status, lim) : -INFINITY;
+                if (TL) {  // timeline only: the moment every logit has arrived
+                    __syncthreads();
+                    if (tid == 0 && t == 0) stamp(kStLogits);
                 }
+                const int k = cta_mass_cut(g, E, a.p, a.rule, cut_sc, cand, a.status, [&](int r, int e, float ge) {
+                    if (TS == 1) {
+                        ulist[r] = e;  // one token: U is its activated set, in rank order
+                        // this CTA's neurons q = b + G i of rank r (q in
+                        // [64 r, 64 r + 64)) are requested right away, into
+                        // slot i, by the thread that activated the expert
+                        if (a.do_ffn) {
+                            const int lo = r * kDExpert;
+                            int q = b, i = 0;
+                            while (q < lo) {
+                                q += G;
+                                i++;
+                            }
+                            for (; q < lo + kDExpert && i < a.NS4; q += G, i++) {
+                                fence_proxy_async_smem();
+                                issue_row(q, i);
+                            }
+                        }
+                    } else {
+                        mask[e] |= 1u << t;
+                    }
+                    const float gv = a.gate == PP_GATE_NONE ? 1.0f : sigmoidf_(ge);
+                    gw[t * E + e] = gv;
+                    if (publish && a.sel_ids) {
+                        a.sel_ids[(size_t)t * E + r] = e;
+                        a.sel_gates[(size_t)t * E + r] = gv;
+                    }
+                }, [&] {
+                    if (TL && tid == 0 && t == 0) stamp(kStCand);
+                });
+                if (tid == 0) s_k[t] = k;
                 if (publish) {
                     if (a.sel_ids)
-                        write_selection_row(a.sel_ids + (size_t)t * E, a.sel_gates + (size_t)t * E, j, E, k, on, r,
-                                            gv);
-                    if (a.sel_logits) a.sel_logits[(size_t)t * E + j] = g;
+                        for (int r = k + tid; r < E; r += kDecThreads) {
+                            a.sel_ids[(size_t)t * E + r] = -1;
+                            a.sel_gates[(size_t)t * E + r] = 0.0f;
+                        }
+                    if (a.sel_logits && tid < E) a.sel_logits[(size_t)t * E + tid] = g;
+                    if (tid == 0 && a.sel_counts) a.sel_counts[t] = k;
                 }
             }
-            if (publish && tid == 0 && a.sel_counts) a.sel_counts[t] = k;
-            __syncthreads();  // scratch reuse by the next token
+            if (TL && tid == 0) stamp(kStCut);
+            // the candidate lists in the ring are dead: order their generic
+            // accesses before the bulk copies into the ring
+            fence_proxy_async_smem();
+        } else {
+            decode_select_cta(a, tag, gw, mask, sel_sc);
         }
     } else {
         load_given_selection(a, gw, mask);
     }
     __syncthreads();
+    if (TL && tid == 0) stamp(kStSelected);
     if (!a.do_ffn) return;
 
     // union U of the tokens' activated experts, ascending expert index
-    {
+    // (already formed, in rank order, by the one-token cut)
+    if (!(a.do_route && mass_cut && TS == 1)) {
         const int e = tid;
         const bool on = e < E && mask[e] != 0u;
         const unsigned bal = __ballot_sync(kFull, on);
@@ -282,7 +397,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
         if (on) ulist[s_wcount[warp] + __popc(bal & ((1u << lane) - 1u))] = e;
         __syncthreads();
     }
-    const int nU = s_nU;
+    const int nU = a.do_route && mass_cut && TS == 1 ? s_k[0] : s_nU;
+    if (TL && tid == 0) stamp(kStUnion);
 
     // phase-6 geometry: CTA b owns rows [r0, r0 + rows) of W_down and y;
     // warp w handles experts u = w + 8 i of U (i < nt_w)
@@ -308,27 +424,13 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     };
 
     // ---------------------------------------------------------- phase 4
+    // neurons are dealt round robin: neuron i of this CTA is global neuron
+    // q = b + G i (neuron q & 63 of the expert at position q >> 6 of U)
     const int Ntot = nU * kDExpert;
-    const int nb = (int)(((long long)b * Ntot) / G);
-    const int ne = (int)(((long long)(b + 1) * Ntot) / G);
-    const int cnt = ne - nb;
-    const uint32_t stage4 = (uint32_t)((gated ? 2 : 1) * rowb);
-    const TW* Wg = reinterpret_cast<const TW*>(a.Wg);
-    const TW* Wu = reinterpret_cast<const TW*>(a.Wu);
-    // neuron i of this CTA (global neuron nb + i) -> ring slot `slot`
-    auto issue4 = [&](int i, int slot) {
-        const int q = nb + i;
-        const size_t row = (size_t)ulist[q >> 6] * kDExpert + (q & 63);
-        unsigned char* dst = ring4 + (size_t)slot * stage4;
-        uint64_t* fb = &bars[kBarFull4 + slot];
-        mbar_arrive_expect_tx(fb, stage4);
-        if (gated) {
-            bulk_g2s(dst, Wg + row * d, (uint32_t)rowb, fb);
-            bulk_g2s(dst + rowb, Wu + row * d, (uint32_t)rowb, fb);
-        } else {
-            bulk_g2s(dst, Wu + row * d, (uint32_t)rowb, fb);
-        }
-    };
+    const int cnt = Ntot > b ? (Ntot - 1 - b) / G + 1 : 0;
+    // the one-token cut has already requested neurons i < min(cnt, NS4)
+    const bool early = a.do_route && mass_cut && TS == 1;
+    auto issue4 = [&](int i, int slot) { issue_row(b + G * i, slot); };
     // dot products of one neuron's gate/up rows (in `slot`) with x over the
     // 16-byte chunks [c0, c1), per token
     auto neuron_dots = [&](int slot, int c0, int c1, float (&au)[TS], float (&ag)[TS]) {
@@ -361,7 +463,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
         }
     };
     auto store_h = [&](int i, int t, float su, float sg) {
-        const int q = nb + i;
+        const int q = b + G * i;
         const int u = q >> 6, n = q & 63;
         const float w = gw[t * E + ulist[u]];
         st_tagged(a.th + ((size_t)u * T + t) * kDExpert + n, tag, w == 0.0f ? 0.0f : act_h(a.act, su, sg) * w);
@@ -371,19 +473,21 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     // warp w streams neurons w, w + NS4, ... through slot w.
     const bool few = cnt > 0 && cnt <= a.NS4;
     const int S = cnt == 1 ? 8 : cnt == 2 ? 4 : cnt <= 4 ? 2 : 1;
-    if (few && tid == 0) {
+    if (few && !early && tid == 0) {
         fence_proxy_async_smem();
         for (int i = 0; i < cnt; i++) issue4(i, i);
     }
-    if (!few && warp < a.NS4 && cnt > warp && lane == 0) {
+    if (!few && !early && warp < a.NS4 && cnt > warp && lane == 0) {
         fence_proxy_async_smem();
         issue4(warp, warp);
     }
+    if (TL && tid == 0) stamp(kStIssued4);
     if (few) {
         if (warp < cnt * S) {
             const int i = warp / S, sl = warp % S;
             const int cs = (nchunk + S - 1) / S;
             mbar_wait(&bars[kBarFull4 + i], 0, a.status, lim);
+            if (TL && tid == 0) stamp(kStLanded4);
             float au[TS], ag[TS];
             neuron_dots(i, sl * cs, min(nchunk, (sl + 1) * cs), au, ag);
 #pragma unroll
@@ -438,9 +542,13 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     }
     // this CTA's phase-4 slots are free again (extra phase-6 slots below)
     __syncthreads();
+    if (TL && tid == 0) stamp(kStPhase4);
 
     // ---------------------------------------------------------- phase 6
-    if (rows == 0) return;
+    if (rows == 0) {
+        if (TL && tid == 0) stamp(kStEnd);
+        return;
+    }
     if (lane == 0) {
         fence_proxy_async_smem();
         for (int i = ded6; i < min(nt_w, slots6); i++) issue6(i);
@@ -492,6 +600,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
                 ready = __all_sync(kFull, ready);
                 if (!ready) __nanosleep(kPollBackoffNs);
             } while (!ready && !__shfl_sync(kFull, (int)poll_give_up(t0, a.status, lim), 0));
+            if (TL && i == 0 && tid == 0) stamp(kStFirstH);
         }
         const unsigned long long* hu = hs_w + (size_t)(i % hch) * hwords;
         float hv[TS][kCPL * kEl];
@@ -534,6 +643,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
             issue6(i + slots6);
         }
     }
+    if (TL && tid == 0) stamp(kStPhase6);
     // reduce over the 8 lanes of a row, then over the warps (fixed order)
 #pragma unroll
     for (int j = 0; j < RPL; j++) {
@@ -555,6 +665,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
             if (w < ntiles) v += red6[(w * R6 + row) * TS + t];
         EL::store(a.y, (size_t)t * d + r0 + row, v);
     }
+    if (TL && tid == 0) stamp(kStEnd);
 }
 
 // ------------------------------------------------------------------ host
@@ -591,8 +702,8 @@ bool decode_plan(const DecodePlanIn& in, DecodePlan* out) {
     const size_t budget = in.smem_limit;
     // dedicated phase-6 slots: 2 per warp when they fit comfortably, else 1
     p.ded6 = (off + 2 * kWarps * stage6 + 2 * stage4 <= budget) ? 2 : 1;
-    p.off_ring6 = (uint32_t)off;
-    off = align_up(off + (size_t)p.ded6 * kWarps * stage6, 1024);
+    p.off_ring6 = (uint32_t)off;  // also the cumulative-mass cut's candidate scratch before phase 6
+    off = align_up(off + std::max((size_t)p.ded6 * kWarps * stage6, (size_t)kWarps * 32 * sizeof(WarpCand)), 1024);
     p.off_ring4 = (uint32_t)off;
     if (off + stage4 > budget) return false;
     const size_t avail = budget - off;
@@ -623,9 +734,10 @@ bool decode_plan(const DecodePlanIn& in, DecodePlan* out) {
     return true;
 }
 
-template <typename TW, int TS, int RPL>
+template <typename TW, int TS, int RPL, bool TL = false>
 static cudaError_t launch_one(const DecodeArgs& a, const DecodePlan& p, int grid, cudaStream_t st) {
-    auto kern = a.chain ? decode_layer_kernel<TW, TS, RPL, true> : decode_layer_kernel<TW, TS, RPL, false>;
+    auto kern = TL ? decode_layer_kernel<TW, TS, RPL, false, true>
+                   : (a.chain ? decode_layer_kernel<TW, TS, RPL, true, false> : decode_layer_kernel<TW, TS, RPL, false, false>);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg{};
@@ -657,6 +769,11 @@ static cudaError_t launch_rpl(const DecodeArgs& a, const DecodePlan& p, int grid
 cudaError_t decode_launch(const DecodeArgs& a, const DecodePlan& p, int dtype, int TS, int grid,
                           cudaStream_t st) {
     if (grid < 1 || grid > kMaxGrid) return cudaErrorInvalidValue;  // one launch count per CTA
+    if (a.tline) {  // the timeline instantiation exists for one bf16 token of a plain layer only
+        if (dtype != PP_BF16 || TS != 1 || a.chain) return cudaErrorInvalidValue;
+        return p.RPL == 8 ? launch_one<__nv_bfloat16, 1, 8, true>(a, p, grid, st)
+                          : launch_one<__nv_bfloat16, 1, 16, true>(a, p, grid, st);
+    }
     if (dtype == PP_BF16) {
         switch (TS) {
             case 1: return launch_rpl<__nv_bfloat16, 1>(a, p, grid, st);

@@ -79,8 +79,11 @@ PP_DEVINL bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // limit_ns.  On expiry records PP_ERR_TIMEOUT and returns false.  A wait
 // that has lasted over 1 ms also gives up as soon as another wait has
 // recorded an error, so one failure cannot chain into many full timeouts.
-PP_DEVINL bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned* status, uint64_t limit_ns) {
-    if (mbar_try_wait(bar, parity)) return true;
+// The bounded loop is a separate (not inlined) function: kernels that run
+// once per launch are bound by instruction fetch, so every call site keeps
+// only the first try_wait inline.
+static __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, unsigned* status,
+                                                   uint64_t limit_ns) {
     const uint64_t t0 = globaltimer_ns();
     while (true) {
         if (mbar_try_wait(bar, parity)) return true;
@@ -91,6 +94,11 @@ PP_DEVINL bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned* status, uint6
         }
         if (dt > 1000000ull && *reinterpret_cast<volatile unsigned*>(status) != 0u) return false;
     }
+}
+
+PP_DEVINL bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned* status, uint64_t limit_ns) {
+    if (mbar_try_wait(bar, parity)) return true;
+    return mbar_wait_slow(bar, parity, status, limit_ns);
 }
 
 // -------------------------------------------------------------------- TMA
@@ -112,6 +120,13 @@ PP_DEVINL void tma_load_2d(void* dst, const CUtensorMap* map, int c0, int c1, ui
         "{%2, %3}], [%4];" ::"r"(smem_u32(dst)),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(smem_u32(bar))
         : "memory");
+}
+
+// 2-D tiled prefetch of a tensor-map box into L2 (no shared memory).
+PP_DEVINL void tma_prefetch_2d(const CUtensorMap* map, int c0, int c1) {
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(map)),
+                 "r"(c0), "r"(c1)
+                 : "memory");
 }
 
 // Programmatic dependent launch: wait until the preceding grid on the stream

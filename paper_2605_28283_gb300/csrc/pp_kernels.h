@@ -56,7 +56,33 @@ struct DecodeArgs {
     const void* gamma;
     void* x_out;
     float eps;
+    // timeline instantiation only: [grid][kDecodeStamps] global-timer stamps
+    unsigned long long* tline;
 };
+
+// Phase boundaries recorded by the decode kernel's timeline instantiation,
+// per CTA (0 where a CTA skips the phase).
+enum DecodeStamp {
+    kStEntry = 0,    // first instruction
+    kStReleased,     // the preceding grid on the stream has completed
+    kStX,            // x (and the launch tag) in shared memory
+    kStRouter,       // this CTA's router logits published
+    kStSelected,     // every token's selection made (all logits received)
+    kStUnion,        // union U of the activated experts formed
+    kStIssued4,      // first gate/up row loads issued
+    kStPhase4,       // this CTA's gate/up activations published
+    kStFirstH,       // warp 0's first activations of phase 6 received
+    kStPhase6,       // warp 0's down-projection products done
+    kStEnd,          // y written (or the CTA's last phase done)
+    kStLogits,       // cumulative-mass cut: every logit of token 0 received (warp 0)
+    kStCut,          // cumulative-mass cut: warp 0's part of the count done
+    kStCand,         // one-warp cut: candidates of token 0 formed (warp 0)
+    kStLanded4,      // warp 0's first gate/up rows landed in shared memory
+    kDecodeStamps = 16
+};
+// SM clock assumed by the timeline stamps between global-timer readings
+// (the maximum clock of this GPU, which it runs at under this load)
+constexpr long long kStampMHz = 2070;
 
 struct DecodePlanIn {
     int dtype, d, E, TS, grid;

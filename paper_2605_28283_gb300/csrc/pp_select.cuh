@@ -405,6 +405,150 @@ PP_DEVINL int cta_select_fn(Load load, int E, float p, int rule, bool want_rank,
     return k;
 }
 
+// ---------------------------------------------------------------------------
+// Cumulative-mass cut of one token (MIN_PREFIX or PAPER with p < 1) by the
+// whole CTA in three barriers, for the fused decode kernel, where every
+// instruction of this serial step is latency.  Thread j holds logit j.  Same
+// arithmetic as cta_select_fn: fp32 max-shifted exponentials summed as exact
+// 2^-31 fixed-point integers; the candidates (a prefix of the order) each get
+// their exclusive prefix mass A and rank counted over the candidates ahead of
+// them; then
+//   MIN_PREFIX: activated <=> A == 0 or A      <= M
+//   PAPER:      activated <=> A == 0 or A + U  <= M
+// with M = prefix_threshold(p, Z) (the largest integer below p Z).  An
+// activated expert carries more than (1 - p) Z / E of the mass (the mass at
+// or behind it exceeds (1 - p) Z and holds at most E exponentials no larger
+// than its own), so the candidates are the experts with
+// g - max >= ln((1 - p) Z' / (2 E)), where Z' is Z to within a few parts in
+// 10^7 (each warp's sum of exp(g - its own max) in 2^-24 fixed point,
+// rescaled to the global max): any Z' below 2 Z keeps every activated
+// expert, and the slack of ln 2 also covers the fast log.
+//   barrier 1: warp maxima (order keys) and approximate sums, non-finite flag
+//   barrier 2: exact warp sums of the fixed-point exponentials; candidates
+//              compacted by one shared atomic per warp
+//   barrier 3: the activated count
+struct WarpCand {
+    unsigned long long key;  // (descending-logit key << 32) | expert index
+    uint32_t U;              // fixed-point exponential
+    float g;                 // logit
+};
+
+struct CutShared {
+    uint32_t wmin[8];  // per warp: smallest order key (its max logit)
+    uint32_t zw[8];    // per warp: sum of exp(g - its max) in 2^-24 units
+    uint32_t zhi[8];   // per warp: sums of the exponentials' high and low 16 bits
+    uint32_t zlo[8];
+    int nc;            // candidates
+};
+
+PP_DEVINL float desc_key_logit(uint32_t D) {
+    const unsigned ord = ~D;
+    return __uint_as_float((ord & 0x80000000u) ? (ord & 0x7fffffffu) : ~ord);
+}
+
+// Every thread of the CTA (8 warps) calls; thread j < E passes logit j.
+// cand: 256 entries of scratch (shared memory).  For every activated expert
+// one thread calls on(rank, expert, logit); every thread calls mid() after
+// barrier 2.  Returns the activated count k, or 0 with PP_ERR_NONFINITE
+// recorded when a logit is not finite.
+template <typename On, typename Mid>
+PP_DEVINL int cta_mass_cut(float g, int E, float p, int rule, CutShared& sc, WarpCand* cand, unsigned* status, On on,
+                           Mid mid) {
+    const int j = threadIdx.x, lane = j & 31, warp = j >> 5;
+    const bool valid = j < E;
+    const bool fin = !valid || isfinite(g);
+    const uint32_t D = valid && fin ? desc_key(g) : 0xffffffffu;
+    const uint32_t wmin = __reduce_min_sync(kFull, D);
+    const float mw = desc_key_logit(wmin);
+    const uint32_t zw = __reduce_add_sync(kFull, valid && fin ? __float2uint_rn(expf(g - mw) * 16777216.0f) : 0u);
+    if (lane == 0) {
+        sc.wmin[warp] = wmin;
+        sc.zw[warp] = zw;
+    }
+    if (j == 0) sc.nc = 0;
+    if (__syncthreads_or(!fin)) {
+        if (j == 0) record_status(status, PP_ERR_NONFINITE);
+        return 0;
+    }
+    uint32_t dmin;
+    {
+        const uint4 a = *reinterpret_cast<const uint4*>(&sc.wmin[0]);
+        const uint4 b = *reinterpret_cast<const uint4*>(&sc.wmin[4]);
+        dmin = min(min(min(a.x, a.y), min(a.z, a.w)), min(min(b.x, b.y), min(b.z, b.w)));
+    }
+    const float m = desc_key_logit(dmin);
+    // sum of exp(g - m) to a few parts in 10^7: lane w < 8 rescales warp w's
+    // sum, three shuffles add the eight terms
+    float zapprox = 0.0f;
+    if (lane < 8) {
+        const uint32_t dw = sc.wmin[lane];
+        if (dw != 0xffffffffu) zapprox = (float)sc.zw[lane] * (1.0f / 16777216.0f) * expf(desc_key_logit(dw) - m);
+    }
+    zapprox += __shfl_xor_sync(kFull, zapprox, 4);
+    zapprox += __shfl_xor_sync(kFull, zapprox, 2);
+    zapprox += __shfl_xor_sync(kFull, zapprox, 1);
+    zapprox = __shfl_sync(kFull, zapprox, 0);
+    const uint32_t U = valid ? __float2uint_rn(expf(g - m) * 2147483648.0f) : 0u;
+    const float Bm = __fdividef((1.0f - fmaxf(p, 0.0f)) * zapprox, (float)E);
+    const float Lc = Bm >= 20.0f / 2147483648.0f ? __logf(0.5f * Bm) : -INFINITY;
+    const bool c = valid && (g - m) >= Lc;
+    const unsigned bal = __ballot_sync(kFull, c);
+    int base = 0;
+    if (lane == 0 && bal) base = atomicAdd(&sc.nc, __popc(bal));
+    base = __shfl_sync(kFull, base, 0);
+    if (c) cand[base + __popc(bal & ((1u << lane) - 1u))] = WarpCand{((unsigned long long)D << 32) | (unsigned)j, U, g};
+    const uint32_t hi = __reduce_add_sync(kFull, U >> 16), lo = __reduce_add_sync(kFull, U & 0xffffu);
+    if (lane == 0) {
+        sc.zhi[warp] = hi;
+        sc.zlo[warp] = lo;
+    }
+    __syncthreads();
+    mid();
+    unsigned long long Z = 0ull;
+#pragma unroll
+    for (int w = 0; w < 8; w++) Z += ((unsigned long long)sc.zhi[w] << 16) + sc.zlo[w];
+    const int nc = sc.nc;
+    const long long thr = prefix_threshold(p, Z);
+    // gs threads per candidate (aligned lane groups), each summing a
+    // contiguous run of the list.  nc <= E <= blockDim and gs * nc <=
+    // blockDim, so a thread takes one candidate at most.
+    int lg = 0;
+    while (lg < 5 && (nc << (lg + 1)) <= (int)blockDim.x) lg++;
+    const int gs = 1 << lg;
+    const int q = j >> lg, part = j & (gs - 1);
+    const bool mine = q < nc;
+    const WarpCand cq = cand[mine ? q : 0];
+    const int per = (nc + gs - 1) >> lg;
+    const int i0 = min(nc, part * per), i1 = min(nc, i0 + per);
+    unsigned long long A0 = 0ull, A1 = 0ull;
+    int r0 = 0, r1 = 0;
+    int i = i0;
+    for (; i + 2 <= i1; i += 2) {
+        const WarpCand c0 = cand[i], c1 = cand[i + 1];
+        const bool a0 = c0.key < cq.key, a1 = c1.key < cq.key;
+        A0 += a0 ? (unsigned long long)c0.U : 0ull;
+        A1 += a1 ? (unsigned long long)c1.U : 0ull;
+        r0 += a0;
+        r1 += a1;
+    }
+    if (i < i1) {
+        const WarpCand c0 = cand[i];
+        const bool a0 = c0.key < cq.key;
+        A0 += a0 ? (unsigned long long)c0.U : 0ull;
+        r0 += a0;
+    }
+    unsigned long long A = A0 + A1;
+    int r = r0 + r1;
+    for (int o = 1; o < gs; o <<= 1) {
+        A += __shfl_xor_sync(kFull, A, o);
+        r += __shfl_xor_sync(kFull, r, o);
+    }
+    const unsigned long long mass = rule == PP_SEL_PAPER ? A + cq.U : A;
+    const bool act = mine && part == 0 && (A == 0ull || (thr >= 0 && mass <= (unsigned long long)thr));
+    if (act) on(r, (int)(unsigned)(cq.key & 0xffffffffull), cq.g);
+    return __syncthreads_count(act);
+}
+
 // The rank-order selection row of one token from cta_select_fn's results
 // (called by every thread j < E): activated experts at their ranks, -1 and
 // gate 0 in the slots k .. E-1.
