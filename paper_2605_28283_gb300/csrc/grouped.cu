@@ -192,6 +192,33 @@ __global__ void __launch_bounds__(256) select_part_cta_kernel(const float* __res
     if (j == 0) counts[t] = k;
 }
 
+// Cumulative-mass cut (MIN_PREFIX / PAPER with p < 1) of any number of
+// tokens: one CTA per token runs the three-barrier cut of the fused decode
+// kernel on the summed partial logits.
+__global__ void __launch_bounds__(256) select_part_cut_kernel(const float* __restrict__ part, int nsplit, int T, int E,
+                                                              float p, int rule, int gate, int32_t* ids,
+                                                              int32_t* counts, float* gates, float* logits_out,
+                                                              unsigned* status) {
+    pdl_wait();  // the previous kernel on the stream has completed (programmatic dependent launch)
+    pdl_launch_dependents();
+    __shared__ __align__(16) CutShared sc;
+    __shared__ __align__(16) WarpCand cand[256];
+    const int t = blockIdx.x, j = threadIdx.x;
+    const float g = j < E ? sum_partials(part, nsplit, (size_t)T * E, (size_t)t * E + j) : -INFINITY;
+    int32_t* idr = ids + (size_t)t * E;
+    float* gtr = gates + (size_t)t * E;
+    const int k = cta_mass_cut(g, E, p, rule, sc, cand, status, [&](int r, int e, float ge) {
+        idr[r] = e;
+        gtr[r] = gate == PP_GATE_NONE ? 1.0f : sigmoidf_(ge);
+    }, [] {});
+    for (int r = k + j; r < E; r += 256) {
+        idr[r] = -1;
+        gtr[r] = 0.0f;
+    }
+    if (j < E && logits_out) logits_out[(size_t)t * E + j] = g;
+    if (j == 0) counts[t] = k;
+}
+
 // ================================================================== dispatch
 // bits[t][w]: bit (e % 32) of word e / 32 set when token t activated e;
 // gexp[t][e]: the gate weight of that assignment (gates of a repeated id
@@ -1299,6 +1326,11 @@ cudaError_t grouped_route(const GroupedArgs& a, cudaStream_t st) {
         default: e = launch_router<256>(mx, mwr, a.T, a.E, g.nk, g.kpb, g.nsplit, a.part, a.status, a.timeout_ns, st); break;
     }
     if (e != cudaSuccess) return e;
+    if ((a.rule == PP_SEL_MIN_PREFIX || a.rule == PP_SEL_PAPER) && a.p < 1.0f) {
+        PP_LAUNCH(select_part_cut_kernel, dim3(a.T), dim3(256), 0, st, a.part, g.nsplit, a.T, a.E, a.p, a.rule,
+                  a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status);
+        return cudaGetLastError();
+    }
     if (a.T <= kCtaSelectMaxTokens) {
         PP_LAUNCH(select_part_cta_kernel, dim3(a.T), dim3(256), 0, st, a.part, g.nsplit, a.T, a.E, a.p, a.rule,
             a.gate, a.ids, a.counts, a.gates, a.logits_out, a.status);
