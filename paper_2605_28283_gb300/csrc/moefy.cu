@@ -221,11 +221,13 @@ void distances(const std::vector<float>& F, const std::vector<double>& fnorm, co
 }
 
 // ---------------------------------------------------------------- device
-// One CTA: every entry of perm in [0, dff) and none repeated, else the
-// status word records PP_ERR_INVALID_ARG.  bitmap: dff bits of shared memory.
-__global__ void __launch_bounds__(1024) perm_check_kernel(const int32_t* __restrict__ perm, int dff,
-                                                          unsigned* status) {
-    extern __shared__ unsigned bitmap[];
+constexpr uint64_t kPermTimeoutNs = 2000000000ull;  // bounded waits give up after 2 s
+
+// Every entry of perm in [0, dff) and none repeated, else the status word
+// records PP_ERR_INVALID_ARG (one CTA of 256 threads; bitmap of dff bits in
+// shared memory, dff <= 256 * 64).
+PP_DEVINL void perm_check_cta(const int32_t* __restrict__ perm, int dff, unsigned* status) {
+    __shared__ unsigned bitmap[kMaxExperts * kDExpert / 32];
     const int words = (dff + 31) >> 5;
     for (int w = threadIdx.x; w < words; w += blockDim.x) bitmap[w] = 0u;
     __syncthreads();
@@ -243,61 +245,118 @@ __global__ void __launch_bounds__(1024) perm_check_kernel(const int32_t* __restr
 }
 
 // Rows of W_gate / W_up: out[m][j][:] = in[m][perm[j]][:] (a zero row for an
-// out-of-range entry, which perm_check_kernel reports).  One row per CTA
-// iteration, 16-byte loads and stores; `chunks` = row bytes / 16.
-__global__ void __launch_bounds__(256) permute_rows_kernel(const int32_t* __restrict__ perm, const uint4* in0,
-                                                           const uint4* in1, uint4* out0, uint4* out1, int dff,
-                                                           int nmat, int chunks) {
+// out-of-range entry).  Row-gather CTA `cta` of `ncta` takes rows cta,
+// cta + ncta, ..., kRowsInFlight of them at a time (every thread loads its
+// 16-byte chunk of all of them before storing any), so that enough bytes are
+// in flight per CTA; `chunks` = row bytes / 16.
+constexpr int kRowsInFlight = 2;
+PP_DEVINL void permute_rows_cta(const int32_t* __restrict__ perm, const uint4* in0, const uint4* in1, uint4* out0,
+                                uint4* out1, int dff, int nmat, int chunks, int cta, int ncta) {
     const long long rows = (long long)dff * nmat;
-    for (long long r = blockIdx.x; r < rows; r += gridDim.x) {
-        const int m = (int)(r / dff);
-        const int j = (int)(r - (long long)m * dff);
-        const int src = perm[j];
-        const uint4* in = m == 0 ? in0 : in1;
-        uint4* out = (m == 0 ? out0 : out1) + (size_t)j * chunks;
-        if (src < 0 || src >= dff) {
-            for (int c = threadIdx.x; c < chunks; c += blockDim.x) out[c] = make_uint4(0u, 0u, 0u, 0u);
-            continue;
+    for (long long r0 = cta; r0 < rows; r0 += (long long)ncta * kRowsInFlight) {
+        const uint4* src[kRowsInFlight];
+        uint4* dst[kRowsInFlight];
+#pragma unroll
+        for (int k = 0; k < kRowsInFlight; k++) {
+            const long long r = r0 + (long long)k * ncta;
+            src[k] = nullptr;
+            dst[k] = nullptr;
+            if (r < rows) {
+                const int m = (int)(r / dff);
+                const int j = (int)(r - (long long)m * dff);
+                const int s = perm[j];
+                dst[k] = (m == 0 ? out0 : out1) + (size_t)j * chunks;
+                if (s >= 0 && s < dff) src[k] = (m == 0 ? in0 : in1) + (size_t)s * chunks;
+            }
         }
-        const uint4* row = in + (size_t)src * chunks;
-        for (int c = threadIdx.x; c < chunks; c += blockDim.x) __stcs(out + c, __ldcs(row + c));
+        for (int c = threadIdx.x; c < chunks; c += blockDim.x) {
+            uint4 v[kRowsInFlight];
+#pragma unroll
+            for (int k = 0; k < kRowsInFlight; k++) v[k] = src[k] ? __ldcs(src[k] + c) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+            for (int k = 0; k < kRowsInFlight; k++)
+                if (dst[k]) __stcs(dst[k] + c, v[k]);
+        }
     }
 }
 
-// Columns of W_down [d][dff]: out[r][j] = in[r][perm[j]].  Each CTA keeps
-// perm in shared memory, stages whole rows of W_down there with 16-byte
-// loads and writes the gathered row with 16-byte stores.  TE is the 16-bit
-// or 32-bit element (bit pattern); VEC = 16 / sizeof(TE).
+// The row gather: the last CTA checks perm instead (the gathers do not depend
+// on the check, so it runs beside them).
+__global__ void __launch_bounds__(256) permute_rows_kernel(const int32_t* __restrict__ perm, const uint4* in0,
+                                                           const uint4* in1, uint4* out0, uint4* out1, int dff,
+                                                           int nmat, int chunks, unsigned* status) {
+    if (blockIdx.x == gridDim.x - 1)
+        perm_check_cta(perm, dff, status);
+    else
+        permute_rows_cta(perm, in0, in1, out0, out1, dff, nmat, chunks, (int)blockIdx.x, (int)gridDim.x - 1);
+}
+
+// Columns of W_down [d][dff]: out[r][j] = in[r][perm[j]].  Each column CTA keeps
+// perm in shared memory (16-bit entries, 0xffff for an out-of-range one) and
+// a ring of nbuf whole rows of W_down, filled by 1-D bulk copies: the copy
+// of a later row is in flight while the current one is gathered and written
+// with 16-byte stores.  TE is the 16-bit or 32-bit element (bit pattern);
+// VEC = 16 / sizeof(TE).  Row bytes (dff * sizeof(TE)) are a multiple of 128.
 template <typename TE>
 __global__ void __launch_bounds__(512) permute_cols_kernel(const int32_t* __restrict__ perm, const TE* in, TE* out,
-                                                           int d, int dff) {
+                                                           int d, int dff, int nbuf, unsigned* status) {
     constexpr int VEC = 16 / (int)sizeof(TE);
-    extern __shared__ __align__(16) unsigned char smem[];
-    int* perm_s = reinterpret_cast<int*>(smem);
-    TE* row_s = reinterpret_cast<TE*>(smem + (size_t)dff * 4);
+    extern __shared__ __align__(128) unsigned char smem[];
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);  // nbuf <= 4 mbarriers
+    uint16_t* perm_s = reinterpret_cast<uint16_t*>(smem + 128);
+    TE* ring = reinterpret_cast<TE*>(smem + 128 + (((size_t)dff * 2 + 127) & ~(size_t)127));
+    const uint32_t row_bytes = (uint32_t)((size_t)dff * sizeof(TE));
+    const int G = gridDim.x;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < nbuf; i++) mbar_init(&bars[i], 1);
+        fence_mbar_init();
+    }
     for (int j = threadIdx.x; j < dff; j += blockDim.x) {
         const int v = perm[j];
-        perm_s[j] = (v >= 0 && v < dff) ? v : -1;
+        perm_s[j] = (v >= 0 && v < dff) ? (uint16_t)v : (uint16_t)0xffff;
     }
+    __syncthreads();
+    auto issue = [&](int i) {  // row blockIdx.x + i G -> buffer i % nbuf
+        const int r = blockIdx.x + i * G;
+        uint64_t* bar = &bars[i % nbuf];
+        mbar_arrive_expect_tx(bar, row_bytes);
+        bulk_g2s(ring + (size_t)(i % nbuf) * dff, in + (size_t)r * dff, row_bytes, bar);
+    };
+    if (threadIdx.x == 0)
+        for (int i = 0; i < nbuf && blockIdx.x + i * G < d; i++) issue(i);
     const int chunks = dff / VEC;
-    for (int r = blockIdx.x; r < d; r += gridDim.x) {
-        const uint4* src = reinterpret_cast<const uint4*>(in + (size_t)r * dff);
-        uint4* srow = reinterpret_cast<uint4*>(row_s);
-        __syncthreads();  // perm_s ready; previous row's gather done
-        for (int c = threadIdx.x; c < chunks; c += blockDim.x) srow[c] = __ldcs(src + c);
-        __syncthreads();
+    for (int i = 0; blockIdx.x + i * G < d; i++) {
+        const int r = blockIdx.x + i * G;
+        const TE* row_s = ring + (size_t)(i % nbuf) * dff;
+        mbar_wait(&bars[i % nbuf], (uint32_t)(i / nbuf) & 1u, status, kPermTimeoutNs);
         uint4* dst = reinterpret_cast<uint4*>(out + (size_t)r * dff);
         for (int c = threadIdx.x; c < chunks; c += blockDim.x) {
+            // the chunk's VEC source indices in one shared-memory load
+            union {
+                uint4 v;
+                uint16_t e[8];
+            } pi;
+            if (VEC == 8) {
+                pi.v = reinterpret_cast<const uint4*>(perm_s)[c];
+            } else {
+                const uint2 h = reinterpret_cast<const uint2*>(perm_s)[c];
+                pi.v = make_uint4(h.x, h.y, 0u, 0u);
+            }
             union {
                 uint4 v;
                 TE e[VEC];
             } u;
 #pragma unroll
             for (int v = 0; v < VEC; ++v) {
-                const int s = perm_s[c * VEC + v];
-                u.e[v] = s >= 0 ? row_s[s] : TE(0);
+                const uint16_t s = pi.e[v];
+                u.e[v] = s != 0xffff ? row_s[s] : TE(0);
             }
             __stcs(dst + c, u.v);
+        }
+        __syncthreads();  // every thread is done with this buffer
+        if (threadIdx.x == 0 && blockIdx.x + (i + nbuf) * G < d) {
+            fence_proxy_async_smem();
+            issue(i + nbuf);
         }
     }
 }
@@ -373,21 +432,26 @@ cudaError_t moefy_permute_launch(int dtype, const int32_t* perm, const void* Wg,
                                  void* Wg_out, void* Wu_out, void* Wd_out, int d, int dff, int sms, unsigned* status,
                                  cudaStream_t st) {
     const size_t esz = dtype == PP_BF16 ? 2 : 4;
-    perm_check_kernel<<<1, 1024, (size_t)((dff + 31) / 32) * 4, st>>>(perm, dff, status);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    // gate / up rows
+    // gate / up rows (plus the permutation check in the last CTA)
     const int nmat = Wg ? 2 : 1;
     const int chunks = (int)((size_t)d * esz / 16);
     const long long rows = (long long)dff * nmat;
-    const int grid_rows = (int)std::min<long long>(rows, (long long)sms * 8);
+    const int grid_rows = (int)std::min<long long>(rows, (long long)sms * 8) + 1;
     permute_rows_kernel<<<grid_rows, 256, 0, st>>>(
         perm, static_cast<const uint4*>(Wg ? Wg : Wu), static_cast<const uint4*>(Wu),
-        static_cast<uint4*>(Wg ? Wg_out : Wu_out), static_cast<uint4*>(Wu_out), dff, nmat, chunks);
-    e = cudaGetLastError();
+        static_cast<uint4*>(Wg ? Wg_out : Wu_out), static_cast<uint4*>(Wu_out), dff, nmat, chunks, status);
+    cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    // down columns
-    const size_t smem = (size_t)dff * 4 + (size_t)dff * esz;
+    // down columns: a ring of up to 3 rows per CTA, two CTAs per SM when they fit
+    int dev = 0, optin = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) != cudaSuccess) return e;
+    const size_t row_bytes = (size_t)dff * esz;
+    const size_t fixed = 128 + (((size_t)dff * 2 + 127) & ~(size_t)127);
+    int nbuf = 3;
+    while (nbuf > 1 && fixed + nbuf * row_bytes > (size_t)optin / 2 - 1024) nbuf--;
+    const size_t smem = fixed + nbuf * row_bytes;
+    if (smem > (size_t)optin) return cudaErrorInvalidValue;
     const void* fn = dtype == PP_BF16 ? (const void*)permute_cols_kernel<uint16_t>
                                       : (const void*)permute_cols_kernel<uint32_t>;
     e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -398,10 +462,10 @@ cudaError_t moefy_permute_launch(int dtype, const int32_t* perm, const void* Wg,
     const int grid_cols = std::max(1, std::min(d, sms * std::max(1, per_sm)));
     if (dtype == PP_BF16)
         permute_cols_kernel<uint16_t><<<grid_cols, 512, smem, st>>>(
-            perm, static_cast<const uint16_t*>(Wd), static_cast<uint16_t*>(Wd_out), d, dff);
+            perm, static_cast<const uint16_t*>(Wd), static_cast<uint16_t*>(Wd_out), d, dff, nbuf, status);
     else
         permute_cols_kernel<uint32_t><<<grid_cols, 512, smem, st>>>(
-            perm, static_cast<const uint32_t*>(Wd), static_cast<uint32_t*>(Wd_out), d, dff);
+            perm, static_cast<const uint32_t*>(Wd), static_cast<uint32_t*>(Wd_out), d, dff, nbuf, status);
     return cudaGetLastError();
 }
 
