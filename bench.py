@@ -39,6 +39,8 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="llama2_7b_decode")
     ap.add_argument("--p", type=float, default=0.7)
+    ap.add_argument("--rule", default="min_prefix", choices=["min_prefix", "paper", "topk", "lte"],
+                    help="activation rule of the headline timing (p is k for topk, delta for lte)")
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--pool", type=int, default=0,
                     help="distinct token sets per layer (default 64 for decode batches, 1 for prefill)")
@@ -605,7 +607,7 @@ def main():
     # ---- headline: p = args.p
     pf = float(np.float32(args.p))
     head = measure(pp, w, B, args.p, args.steps, args.warmup, args.pool, args.seed, device, stream, flush, world,
-                   profile_range=True)
+                   rule=args.rule, gate="none" if args.rule == "lte" else "sigmoid", profile_range=True)
     desc, ws, layers = head["desc"], head["ws"], head["layers"]
     value, ms_per_step, roof = head["tokens_per_s"], head["ms_per_step"], head["roofline"]
     head_rec = public(head)

@@ -70,8 +70,7 @@ static __device__ __noinline__ void load_given_selection(const DecodeArgs& a, fl
 // as they arrive, for the rules other than the cumulative-mass cut (top-k,
 // LTE's threshold, p >= 1); CTA 0 publishes it.  Out of line, like
 // load_given_selection.
-static __device__ __noinline__ void decode_select_cta(const DecodeArgs& a, unsigned tag, float* gw, unsigned* mask,
-                                                      CtaSelScratch& sc) {
+PP_DEVINL void decode_select_cta(const DecodeArgs& a, unsigned tag, float* gw, unsigned* mask, CtaSelScratch& sc) {
     const int tid = threadIdx.x, T = a.T, E = a.E;
     const bool publish = blockIdx.x == 0;
     const bool want_rank = publish && a.sel_ids != nullptr;
@@ -128,7 +127,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     unsigned char* ring4 = smem + a.off_ring4;
     unsigned char* ring6 = smem + a.off_ring6;
     __shared__ __align__(16) CtaSelScratch sel_sc;
-    __shared__ __align__(16) CutShared cut_sc;
+    __shared__ __align__(16) CutShared cut_sc[kWarps];  // one per token group of the cut
     __shared__ int s_nU;
     __shared__ int s_wcount[kWarps];
     __shared__ unsigned s_tag;
@@ -309,19 +308,28 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
         if (TL && tid == 0) stamp(kStRouter);
         const bool publish = b == 0;
         if (mass_cut) {
-            // cumulative-mass cut of every token by the whole CTA (thread j
-            // waits for logit j); every activated expert is recorded by the
-            // thread that decides it
-            // candidate scratch in the phase-6 ring, idle until phase 6: the
-            // phase-4 ring takes gate/up rows requested during the count
-            WarpCand* cand = reinterpret_cast<WarpCand*>(ring6);
-            for (int t = 0; t < T; t++) {
-                const float g = tid < E ? wait_tagged(a.tlog + (size_t)t * E + tid, tag, a.status, lim) : -INFINITY;
+            // cumulative-mass cut of every token: the tokens are cut side by
+            // side by groups of nt threads (the smallest of 32, 64, 128, 256
+            // that holds E experts; up to TS groups, each with its own named
+            // barrier); thread j of a group waits for logit j of its token,
+            // and every activated expert is recorded by the thread that
+            // decides it.  Candidate scratch in the phase-6 ring, idle until
+            // phase 6 (the phase-4 ring takes gate/up rows requested during
+            // the count).
+            const int nt = E <= 32 ? 32 : E <= 64 ? 64 : E <= 128 ? 128 : kDecThreads;
+            const int ng = min(TS, kDecThreads / nt);
+            const int grp = tid / nt, gj = tid % nt;
+            const int bid = nt == kDecThreads ? 0 : 1 + grp;
+            WarpCand* cand = reinterpret_cast<WarpCand*>(ring6) + (size_t)grp * nt;
+            for (int t0 = 0; t0 < T; t0 += ng) {
+                const int t = t0 + grp;
+                if (grp >= ng || t >= T) continue;
+                const float g = gj < E ? wait_tagged(a.tlog + (size_t)t * E + gj, tag, a.status, lim) : -INFINITY;
                 if (TL) {  // timeline only: the moment every logit has arrived
-                    __syncthreads();
+                    group_bar(bid, nt);
                     if (tid == 0 && t == 0) stamp(kStLogits);
                 }
-                const int k = cta_mass_cut(g, E, a.p, a.rule, cut_sc, cand, a.status, [&](int r, int e, float ge) {
+                const int k = group_mass_cut(g, E, a.p, a.rule, cut_sc[grp], cand, a.status, bid, nt, [&](int r, int e, float ge) {
                     if (TS == 1) {
                         ulist[r] = e;  // one token: U is its activated set, in rank order
                         // this CTA's neurons q = b + G i of rank r (q in
@@ -340,7 +348,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
                             }
                         }
                     } else {
-                        mask[e] |= 1u << t;
+                        atomicOr(&mask[e], 1u << t);  // tokens of other groups at the same time
                     }
                     const float gv = a.gate == PP_GATE_NONE ? 1.0f : sigmoidf_(ge);
                     gw[t * E + e] = gv;
@@ -351,15 +359,15 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
                 }, [&] {
                     if (TL && tid == 0 && t == 0) stamp(kStCand);
                 });
-                if (tid == 0) s_k[t] = k;
+                if (gj == 0) s_k[t] = k;
                 if (publish) {
                     if (a.sel_ids)
-                        for (int r = k + tid; r < E; r += kDecThreads) {
+                        for (int r = k + gj; r < E; r += nt) {
                             a.sel_ids[(size_t)t * E + r] = -1;
                             a.sel_gates[(size_t)t * E + r] = 0.0f;
                         }
-                    if (a.sel_logits && tid < E) a.sel_logits[(size_t)t * E + tid] = g;
-                    if (tid == 0 && a.sel_counts) a.sel_counts[t] = k;
+                    if (a.sel_logits && gj < E) a.sel_logits[(size_t)t * E + gj] = g;
+                    if (gj == 0 && a.sel_counts) a.sel_counts[t] = k;
                 }
             }
             if (TL && tid == 0) stamp(kStCut);

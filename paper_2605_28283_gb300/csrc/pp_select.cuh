@@ -446,15 +446,43 @@ PP_DEVINL float desc_key_logit(uint32_t D) {
     return __uint_as_float((ord & 0x80000000u) ? (ord & 0x7fffffffu) : ~ord);
 }
 
-// Every thread of the CTA (8 warps) calls; thread j < E passes logit j.
-// cand: 256 entries of scratch (shared memory).  For every activated expert
-// one thread calls on(rank, expert, logit); every thread calls mid() after
-// barrier 2.  Returns the activated count k, or 0 with PP_ERR_NONFINITE
-// recorded when a logit is not finite.
+// Barriers of a group of nt threads (whole warps) with barrier id `id`
+// (id 0 with the whole CTA is __syncthreads).
+PP_DEVINL void group_bar(int id, int nt) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nt) : "memory"); }
+PP_DEVINL bool group_bar_or(int id, int nt, bool v) {
+    unsigned r;
+    asm volatile(
+        "{\n\t.reg .pred pi, po;\n\t"
+        "setp.ne.u32 pi, %1, 0;\n\t"
+        "bar.red.or.pred po, %2, %3, pi;\n\t"
+        "selp.u32 %0, 1, 0, po;\n\t}"
+        : "=r"(r)
+        : "r"((unsigned)v), "r"(id), "r"(nt)
+        : "memory");
+    return r != 0u;
+}
+PP_DEVINL int group_bar_count(int id, int nt, bool v) {
+    unsigned r;
+    asm volatile(
+        "{\n\t.reg .pred pi;\n\t"
+        "setp.ne.u32 pi, %1, 0;\n\t"
+        "bar.red.popc.u32 %0, %2, %3, pi;\n\t}"
+        : "=r"(r)
+        : "r"((unsigned)v), "r"(id), "r"(nt)
+        : "memory");
+    return (int)r;
+}
+
+// Every thread of a group of nt = 32 w threads (w <= 8 whole warps, nt >= E)
+// calls, with the group's barrier id; thread j < E of the group passes logit
+// j.  cand: nt entries of scratch (shared memory); sc: the group's own.  For
+// every activated expert one thread calls on(rank, expert, logit); every
+// thread calls mid() after barrier 2.  Returns the activated count k, or 0
+// with PP_ERR_NONFINITE recorded when a logit is not finite.
 template <typename On, typename Mid>
-PP_DEVINL int cta_mass_cut(float g, int E, float p, int rule, CutShared& sc, WarpCand* cand, unsigned* status, On on,
-                           Mid mid) {
-    const int j = threadIdx.x, lane = j & 31, warp = j >> 5;
+PP_DEVINL int group_mass_cut(float g, int E, float p, int rule, CutShared& sc, WarpCand* cand, unsigned* status,
+                             int bid, int nt, On on, Mid mid) {
+    const int j = threadIdx.x & (nt - 1), lane = j & 31, warp = j >> 5, nw = nt >> 5;
     const bool valid = j < E;
     const bool fin = !valid || isfinite(g);
     const uint32_t D = valid && fin ? desc_key(g) : 0xffffffffu;
@@ -466,21 +494,19 @@ PP_DEVINL int cta_mass_cut(float g, int E, float p, int rule, CutShared& sc, War
         sc.zw[warp] = zw;
     }
     if (j == 0) sc.nc = 0;
-    if (__syncthreads_or(!fin)) {
+    if (group_bar_or(bid, nt, !fin)) {
         if (j == 0) record_status(status, PP_ERR_NONFINITE);
         return 0;
     }
-    uint32_t dmin;
-    {
-        const uint4 a = *reinterpret_cast<const uint4*>(&sc.wmin[0]);
-        const uint4 b = *reinterpret_cast<const uint4*>(&sc.wmin[4]);
-        dmin = min(min(min(a.x, a.y), min(a.z, a.w)), min(min(b.x, b.y), min(b.z, b.w)));
-    }
+    uint32_t dmin = 0xffffffffu;  // (loops unrolled to 8 so that the loads issue together)
+#pragma unroll
+    for (int w = 0; w < 8; w++)
+        if (w < nw) dmin = min(dmin, sc.wmin[w]);
     const float m = desc_key_logit(dmin);
-    // sum of exp(g - m) to a few parts in 10^7: lane w < 8 rescales warp w's
-    // sum, three shuffles add the eight terms
+    // sum of exp(g - m) to a few parts in 10^7: lane w < nw rescales warp w's
+    // sum, three shuffles add the (up to eight) terms
     float zapprox = 0.0f;
-    if (lane < 8) {
+    if (lane < nw) {
         const uint32_t dw = sc.wmin[lane];
         if (dw != 0xffffffffu) zapprox = (float)sc.zw[lane] * (1.0f / 16777216.0f) * expf(desc_key_logit(dw) - m);
     }
@@ -502,18 +528,19 @@ PP_DEVINL int cta_mass_cut(float g, int E, float p, int rule, CutShared& sc, War
         sc.zhi[warp] = hi;
         sc.zlo[warp] = lo;
     }
-    __syncthreads();
+    group_bar(bid, nt);
     mid();
     unsigned long long Z = 0ull;
 #pragma unroll
-    for (int w = 0; w < 8; w++) Z += ((unsigned long long)sc.zhi[w] << 16) + sc.zlo[w];
+    for (int w = 0; w < 8; w++)
+        if (w < nw) Z += ((unsigned long long)sc.zhi[w] << 16) + sc.zlo[w];
     const int nc = sc.nc;
     const long long thr = prefix_threshold(p, Z);
     // gs threads per candidate (aligned lane groups), each summing a
-    // contiguous run of the list.  nc <= E <= blockDim and gs * nc <=
-    // blockDim, so a thread takes one candidate at most.
+    // contiguous run of the list.  nc <= E <= nt and gs * nc <= nt, so a
+    // thread takes one candidate at most.
     int lg = 0;
-    while (lg < 5 && (nc << (lg + 1)) <= (int)blockDim.x) lg++;
+    while (lg < 5 && (nc << (lg + 1)) <= nt) lg++;
     const int gs = 1 << lg;
     const int q = j >> lg, part = j & (gs - 1);
     const bool mine = q < nc;
@@ -546,7 +573,14 @@ PP_DEVINL int cta_mass_cut(float g, int E, float p, int rule, CutShared& sc, War
     const unsigned long long mass = rule == PP_SEL_PAPER ? A + cq.U : A;
     const bool act = mine && part == 0 && (A == 0ull || (thr >= 0 && mass <= (unsigned long long)thr));
     if (act) on(r, (int)(unsigned)(cq.key & 0xffffffffull), cq.g);
-    return __syncthreads_count(act);
+    return group_bar_count(bid, nt, act);
+}
+
+// The whole CTA (8 warps) on one token.
+template <typename On, typename Mid>
+PP_DEVINL int cta_mass_cut(float g, int E, float p, int rule, CutShared& sc, WarpCand* cand, unsigned* status, On on,
+                           Mid mid) {
+    return group_mass_cut(g, E, p, rule, sc, cand, status, 0, 256, on, mid);
 }
 
 // The rank-order selection row of one token from cta_select_fn's results
