@@ -157,10 +157,19 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     if (tid < TS) s_k[tid] = 0;
     __syncthreads();
 
-    // this CTA's router rows [j0, j1) of W_r (phase 1)
+    // this CTA's router rows of W_r (phase 1): the E rows form blocks of rpc
+    // rows, and block j is computed by two CTAs, j and (j + G/2) mod G; they
+    // publish the same value, and a reader takes whichever copy arrives first
+    // (a CTA that starts late then delays no logit)
     const int rpc = (E + G - 1) / G;
-    const int j0 = b * rpc, j1 = min(E, j0 + rpc);
-    const int nrows = a.do_route ? max(0, j1 - j0) : 0;
+    const int nblk = (E + rpc - 1) / rpc;
+    const int blkA = b < nblk ? b : -1;
+    const int bB = (b + G / 2) % G;
+    const int blkB = bB < nblk && bB != blkA ? bB : -1;
+    const int jA = blkA * rpc, jB = blkB * rpc;
+    const int nA = a.do_route && blkA >= 0 ? min(E, jA + rpc) - jA : 0;
+    const int nB = a.do_route && blkB >= 0 ? min(E, jB + rpc) - jB : 0;
+    const int nrows = nA + nB;
 
     // The router rows are weights: load them before waiting for the
     // preceding grid (with programmatic dependent launch this overlaps the
@@ -168,9 +177,9 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
     // or scratch, so they are touched only after the wait.
     if (tid == 0 && nrows > 0) {
         const TW* wr = reinterpret_cast<const TW*>(a.Wr);
-        const uint32_t rbytes = (uint32_t)(nrows * rowb);
-        mbar_arrive_expect_tx(&bars[kBarR], rbytes);
-        bulk_g2s(ring4, wr + (size_t)j0 * d, rbytes, &bars[kBarR]);
+        mbar_arrive_expect_tx(&bars[kBarR], (uint32_t)(nrows * rowb));
+        if (nA > 0) bulk_g2s(ring4, wr + (size_t)jA * d, (uint32_t)(nA * rowb), &bars[kBarR]);
+        if (nB > 0) bulk_g2s(ring4 + (size_t)nA * rowb, wr + (size_t)jB * d, (uint32_t)(nB * rowb), &bars[kBarR]);
     }
     pdl_wait();
     pdl_launch_dependents();
@@ -299,7 +308,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_layer_kernel(const __gr
                     if (r0 + i < nrows && t < T) {
                         float v = 0.0f;
                         for (int w = 0; w < kWarps; w++) v += red[(w * 2 + i) * TS + t];
-                        st_tagged(a.tlog + (size_t)t * E + j0 + r0 + i, tag, v);
+                        const int ri = r0 + i;
+                        st_tagged(a.tlog + (size_t)t * E + (ri < nA ? jA + ri : jB + ri - nA), tag, v);
                     }
                 }
                 __syncthreads();
@@ -717,9 +727,9 @@ bool decode_plan(const DecodePlanIn& in, DecodePlan* out) {
     const size_t avail = budget - off;
     // the ring also stages the router rows and, for a chained step, y_prev
     // [TS][d] and gamma [d] (all read before phase 4 uses the ring)
-    p.off_chain = (uint32_t)align_up((size_t)rpc * in.d * esz, 128);
+    p.off_chain = (uint32_t)align_up((size_t)2 * rpc * in.d * esz, 128);  // up to two blocks of router rows
     const size_t chain_end =
-        in.chain ? (size_t)p.off_chain + align_up((size_t)(TS + 1) * in.d * esz, 128) : (size_t)rpc * in.d * esz;
+        in.chain ? (size_t)p.off_chain + align_up((size_t)(TS + 1) * in.d * esz, 128) : (size_t)2 * rpc * in.d * esz;
     const int ns4 = (int)std::min<size_t>(kMaxNS4, avail / stage4);
     // the ring also holds this CTA's router rows (phase 1) and, once phase 4
     // is done, the extra phase-6 slots plus at least one expert's h per warp

@@ -505,3 +505,33 @@ def test_workspace_reuse_across_calls(pp):
         for a, b in zip(got, want):
             assert np.array_equal(a, b), (kind, T, p)
         assert pp.pp_get_device_status(shared) == pp.PP_OK
+
+
+def test_decode_timeline_entry_point(pp):
+    """pp_debug_decode_timeline runs the timeline instantiation of the fused
+    decode kernel: the same y as pp_layer, bitwise (the stamps only add
+    stores), and for every CTA the recorded phase boundaries are ordered in
+    time (entry, release, x loaded, router published, selection made)."""
+    import torch
+    w, L = layer_inputs("llama2_7b_decode", 1)
+    desc = pp.make_desc(w.d_model, w.n_experts, w.dtype, w.act)
+    ws = pp.alloc_workspace(desc, 1)
+    args = [dev(a) for a in (L.x, L.Wr, L.Wg, L.Wu, L.Wd)]
+    y_ref = torch.empty_like(args[0])
+    pp.pp_layer(desc, args[0], 1, *args[1:], f32(0.7), None, y_ref, ws)
+    stamps = torch.zeros(256 * 16, dtype=torch.int64, device="cuda")
+    y = torch.empty_like(args[0])
+    pp.pp_debug_decode_timeline(desc, args[0], *args[1:], f32(0.7), y, ws, stamps)
+    torch.cuda.synchronize()
+    assert pp.pp_get_device_status(ws) == pp.PP_OK
+    assert torch.equal(y.view(torch.int16), y_ref.view(torch.int16))
+    sm = torch.cuda.get_device_properties(0).multi_processor_count
+    st = stamps.view(256, 16)[:sm].cpu().numpy()
+    assert np.all(st[:, 0] > 0)  # every CTA stamped its entry
+    for i in range(1, 5):  # entry <= released <= x <= router <= selected
+        assert np.all(st[:, i] >= st[:, i - 1]), i
+    # the timeline exists for one bf16 token only
+    d32 = pp.make_desc(256, 16, "f32", "relu")
+    with pytest.raises(pp.PPError) as ei:
+        pp.pp_debug_decode_timeline(d32, args[0], *args[1:], 0.7, y, ws, stamps)
+    assert ei.value.status == pp.PP_ERR_DTYPE
