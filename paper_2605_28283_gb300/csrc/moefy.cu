@@ -285,6 +285,7 @@ PP_DEVINL void permute_rows_cta(const int32_t* __restrict__ perm, const uint4* i
 __global__ void __launch_bounds__(256) permute_rows_kernel(const int32_t* __restrict__ perm, const uint4* in0,
                                                            const uint4* in1, uint4* out0, uint4* out1, int dff,
                                                            int nmat, int chunks, unsigned* status) {
+    pdl_launch_dependents();  // the column gather (next on the stream) does not read what this grid writes
     if (blockIdx.x == gridDim.x - 1)
         perm_check_cta(perm, dff, status);
     else
@@ -359,6 +360,9 @@ __global__ void __launch_bounds__(512) permute_cols_kernel(const int32_t* __rest
             issue(i + nbuf);
         }
     }
+    // started beside the row gather (programmatic dependent launch): finish
+    // only after it, so that work later on the stream sees both
+    pdl_wait();
 }
 
 }  // namespace
@@ -460,12 +464,25 @@ cudaError_t moefy_permute_launch(int dtype, const int32_t* perm, const void* Wg,
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, 512, smem);
     if (e != cudaSuccess) return e;
     const int grid_cols = std::max(1, std::min(d, sms * std::max(1, per_sm)));
+    // launched with programmatic dependent launch: it runs beside the row
+    // gather (bound by DRAM) while it is bound by shared memory
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(grid_cols);
+    cfg.blockDim = dim3(512);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
     if (dtype == PP_BF16)
-        permute_cols_kernel<uint16_t><<<grid_cols, 512, smem, st>>>(
-            perm, static_cast<const uint16_t*>(Wd), static_cast<uint16_t*>(Wd_out), d, dff, nbuf, status);
+        e = cudaLaunchKernelEx(&cfg, permute_cols_kernel<uint16_t>, perm, static_cast<const uint16_t*>(Wd),
+                               static_cast<uint16_t*>(Wd_out), d, dff, nbuf, status);
     else
-        permute_cols_kernel<uint32_t><<<grid_cols, 512, smem, st>>>(
-            perm, static_cast<const uint32_t*>(Wd), static_cast<uint32_t*>(Wd_out), d, dff, nbuf, status);
+        e = cudaLaunchKernelEx(&cfg, permute_cols_kernel<uint32_t>, perm, static_cast<const uint32_t*>(Wd),
+                               static_cast<uint32_t*>(Wd_out), d, dff, nbuf, status);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
