@@ -1132,7 +1132,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             // token of assignment row a0 + lane (for rows past ycap)
             const long long arow_l = (long long)w.a0 + lane;
             const int tok_l = lane < w.cnt && arow_l >= ycap ? perm_token[arow_l] : -1;
-            if (lane == 0 && (long long)w.a0 + w.cnt > ycap) *overflow = 1;
+            const bool spill = (long long)w.a0 + w.cnt > ycap;  // some of the item's rows go to yacc
+            if (lane == 0 && spill) *overflow = 1;
             for (int rt = r0; rt < r1; rt++, acc++) {
                 const int a = acc & 1;
                 mbar_wait(&tfull[a], (uint32_t)(acc >> 1) & 1u, status, lim);
@@ -1144,15 +1145,26 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&tempty[a]);
                 const int row = rt * 128 + 32 * q + lane;  // output element of d
+                if (!spill) {  // every row of the item is kept: only its cnt columns are stored
+                    if (row < d) {
+                        __nv_bfloat16* yp = Y + (size_t)w.a0 * d + row;
 #pragma unroll
-                for (int t = 0; t < kSwN; t++) {
-                    const int tk = __shfl_sync(kFull, tok_l, t);
-                    if (t < w.cnt && row < d) {
-                        const long long arow = (long long)w.a0 + t;
-                        if (arow < ycap)
-                            Y[(size_t)arow * d + row] = __float2bfloat16_rn(__uint_as_float(val[t]));
-                        else
-                            atomicAdd(&yacc[(size_t)tk * d + row], __uint_as_float(val[t]));
+                        for (int t = 0; t < kSwN; t++) {
+                            if (t >= w.cnt) break;
+                            yp[(size_t)t * d] = __float2bfloat16_rn(__uint_as_float(val[t]));
+                        }
+                    }
+                } else {
+#pragma unroll
+                    for (int t = 0; t < kSwN; t++) {
+                        const int tk = __shfl_sync(kFull, tok_l, t);
+                        if (t < w.cnt && row < d) {
+                            const long long arow = (long long)w.a0 + t;
+                            if (arow < ycap)
+                                Y[(size_t)arow * d + row] = __float2bfloat16_rn(__uint_as_float(val[t]));
+                            else
+                                atomicAdd(&yacc[(size_t)tk * d + row], __uint_as_float(val[t]));
+                        }
                     }
                 }
             }
