@@ -413,15 +413,39 @@ __global__ void __launch_bounds__(1024) dispatch_small_kernel(const int32_t* __r
     }
     if (tid == 0) *overflow = 0;
     __syncthreads();
-    // token masks: warp w takes tokens w, w + 32, ...; lane r its entries
-    for (int t = warp; t < T; t += 32) {
-        int k = counts[t];
+    // warp w takes tokens w + 32 i, lane r their entries r, r + 32, ...; the
+    // count and entry r = lane of each of the warp's tokens are read once, all
+    // loads independent (the three passes below reuse them)
+    constexpr int kTokPerWarp = kSmallDispatchMaxT / 32;
+    int ck[kTokPerWarp], ce[kTokPerWarp];
+    float cg[kTokPerWarp];
+#pragma unroll
+    for (int i = 0; i < kTokPerWarp; i++) {
+        const int t = warp + 32 * i;
+        ck[i] = 0;
+        ce[i] = -1;
+        cg[i] = 0.0f;
+        if (t < T) {
+            ck[i] = counts[t];
+            if (lane < E) {
+                ce[i] = ids[(size_t)t * E + lane];
+                cg[i] = gates[(size_t)t * E + lane];
+            }
+        }
+    }
+    // token masks
+#pragma unroll
+    for (int i = 0; i < kTokPerWarp; i++) {
+        const int t = warp + 32 * i;
+        if (t >= T) break;
+        int k = ck[i];
         if (k < 0 || k > E) {
             if (lane == 0) record_status(status, PP_ERR_INVALID_ARG);
             k = k < 0 ? 0 : E;
         }
+        ck[i] = k;
         for (int r = lane; r < k; r += 32) {
-            const int e = ids[(size_t)t * E + r];
+            const int e = r == lane ? ce[i] : ids[(size_t)t * E + r];
             if (e < 0 || e >= E) {
                 record_status(status, PP_ERR_INVALID_ARG);
                 continue;
@@ -489,16 +513,19 @@ __global__ void __launch_bounds__(1024) dispatch_small_kernel(const int32_t* __r
     // scatter: the first entry of each (t, e) writes its slot, repeats add
     // their gate afterwards
     for (int pass = 0; pass < 2; pass++) {
-        for (int t = warp; t < T; t += 32) {
-            const int k = min(max(counts[t], 0), E);
+#pragma unroll
+        for (int i = 0; i < kTokPerWarp; i++) {
+            const int t = warp + 32 * i;
+            if (t >= T) break;
+            const int k = ck[i];
             for (int r = lane; r < k; r += 32) {
-                const int e = ids[(size_t)t * E + r];
+                const int e = r == lane ? ce[i] : ids[(size_t)t * E + r];
                 if (e < 0 || e >= E) continue;
                 const bool rep = (dup[t][r >> 5] >> (r & 31)) & 1u;
                 if (rep != (pass == 1)) continue;
                 int pos = off_s[e] + __popc(mask[e][t >> 5] & ((1u << (t & 31)) - 1u));
                 for (int w = 0; w < (t >> 5); w++) pos += __popc(mask[e][w]);
-                const float gv = gates[(size_t)t * E + r];
+                const float gv = r == lane ? cg[i] : gates[(size_t)t * E + r];
                 if (pass == 0) {
                     perm_token[pos] = t;
                     perm_gate[pos] = gv;
