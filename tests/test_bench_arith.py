@@ -83,3 +83,18 @@ def test_peaks_fallback_without_measured_file(tmp_path, monkeypatch):
     (tmp_path / "MEASURED_PEAKS.json").write_text(json.dumps({"hbm_gbs": 6778.0, "bf16_tflops": 1940.4,
                                                               "bf16_tflops_sustained": 1695.3}))
     assert bench.load_peaks() == (6778.0, 1695.3, "measured")
+
+
+def test_default_benchmark_lines_have_current_traffic_records(monkeypatch):
+    """Every workload the default bench run reports (the headline and its
+    configs) has a DRAM-traffic record taken at the current kernel sources, so
+    its roofline line carries measured traffic rather than null."""
+    monkeypatch.setattr("sys.argv", ["bench.py"])
+    args = bench.parse()
+    runs = [(args.workload, args.p, args.batch)]
+    for item in [v for v in args.configs.split(",") if v]:
+        parts = item.split(":")
+        runs.append((parts[0], float(parts[2]), int(parts[1])))
+    for name, p, b in runs:
+        kind = bench.path_kind(W[name], b)
+        assert bench.kernel_traffic(name, p, b, kind) is not None, (name, p, b, kind)
